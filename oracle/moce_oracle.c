@@ -1,0 +1,399 @@
+/*
+ * MoCE layer forward: CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY. This file is a plain, slow, double-precision
+ * restatement of the Mixture of Channel Experts layer of "Mixture of Channel
+ * Experts: Static Sparse Supports with Input-Adaptive Mixing for Pointwise
+ * Projections" (Sec. 3). Only the tests, the smoke check and the benchmark's
+ * CPU-baseline leg load it. The CUDA library never calls it and shares no code,
+ * header, table or helper with it.
+ *
+ * Every step follows the paper's definitions in the paper's order, with no
+ * blocking, fusion or reordering:
+ *   support   Eq. (support), Sec. 3.2      S_e = TopK(L_e, k)
+ *   packing   Sec. 3.5 "Storage", Sec. 3.3  keep the k selected (index, logit)
+ *             pairs per expert, ordered by descending logit (the gate input is
+ *             positional, Sec. 3.3)
+ *   pooling   Sec. 3.3                      z = GAP(X)
+ *   gate      Eq. (tau), Sec. 3.3; shape from Sec. 4.1 (two-layer MLP, hidden
+ *             width k, ReLU, biases)
+ *   weights   Eq. (weights)                 a = softmax(L_S / tau)
+ *   routed    Eq. (expert)                  Y_e = sum_i a_i X_i
+ *   residual  Eq. (res), Sec. 3.4           mean of X over U, 0 if U is empty
+ *
+ * Readings where the paper is silent (each is listed in the design notes):
+ *   - ties between equal logits order by ascending channel index; -0.0 and
+ *     +0.0 compare equal; non-finite logits are rejected;
+ *   - the gate is h = ReLU(W1 u + b1) with W1 stored row-major [hidden][input],
+ *     g = w2 . h + b2, sigma is the logistic function;
+ *   - the softmax subtracts the largest support logit before exponentiating,
+ *     which leaves Eq. (weights) unchanged;
+ *   - U is listed in ascending channel order.
+ *
+ * Inputs are the exact values the device sees (bf16 inputs are decoded to
+ * float first); all arithmetic is in double.
+ *
+ * Layouts: 0 = NHWC (channel fastest), 1 = NCHW (pixel fastest). The output y
+ * has R + 1 channels in the same layout, the residual expert last.
+ */
+#include <math.h>
+#include <stddef.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_OK 0
+#define ORACLE_BAD_ARG 1
+#define ORACLE_BAD_SUPPORT 2
+#define ORACLE_NO_MEMORY 3
+
+static size_t x_at(int layout, int n, int p, int c, int HW, int C)
+{
+    if (layout == 0)
+        return ((size_t)n * HW + p) * (size_t)C + c;
+    return ((size_t)n * C + c) * (size_t)HW + p;
+}
+
+/* One (channel, logit) pair of an expert's support. */
+typedef struct {
+    int32_t idx;
+    float logit;
+} oracle_pair;
+
+/* Deployment order: larger logit first; equal logits by smaller channel. */
+static int pair_order(const void *pa, const void *pb)
+{
+    const oracle_pair *a = (const oracle_pair *)pa;
+    const oracle_pair *b = (const oracle_pair *)pb;
+    if (a->logit > b->logit)
+        return -1;
+    if (a->logit < b->logit)
+        return 1;
+    return (a->idx > b->idx) - (a->idx < b->idx);
+}
+
+/*
+ * Eq. (support): S_e = TopK(L_e, k) over a full routing row L_e in R^C.
+ * L is [R][C]. Writes the k selected channels and their logits per expert,
+ * already in deployment order.
+ */
+int moce_oracle_topk(int C, int R, int k, const float *L, int32_t *idx_out, float *logit_out)
+{
+    if (C < 1 || R < 1 || k < 1 || k > C || !L || !idx_out || !logit_out)
+        return ORACLE_BAD_ARG;
+    oracle_pair *row = (oracle_pair *)malloc(sizeof(oracle_pair) * (size_t)C);
+    if (!row)
+        return ORACLE_NO_MEMORY;
+    for (int e = 0; e < R; ++e) {
+        for (int c = 0; c < C; ++c) {
+            float v = L[(size_t)e * C + c];
+            if (!isfinite(v)) {
+                free(row);
+                return ORACLE_BAD_SUPPORT;
+            }
+            row[c].idx = c;
+            row[c].logit = v;
+        }
+        qsort(row, (size_t)C, sizeof(oracle_pair), pair_order);
+        for (int i = 0; i < k; ++i) {
+            idx_out[(size_t)e * k + i] = row[i].idx;
+            logit_out[(size_t)e * k + i] = row[i].logit;
+        }
+    }
+    free(row);
+    return ORACLE_OK;
+}
+
+/*
+ * Deployment packing (Sec. 3.5 "Storage"; order rule of Sec. 3.3; U of
+ * Sec. 3.4). support_idx / support_logits are [R][k] in any row order.
+ * Outputs: each row sorted into deployment order, the unselected channels U
+ * in ascending order (resid, capacity C) and |U|.
+ * A support index outside [0, C), a repeated index within one expert, or a
+ * non-finite logit is rejected.
+ */
+int moce_oracle_pack(int C, int R, int k, const int32_t *support_idx, const float *support_logits,
+                     int32_t *packed_idx, float *packed_logits, int32_t *resid, int32_t *n_resid)
+{
+    if (C < 1 || R < 1 || k < 1 || k > C || !support_idx || !support_logits || !packed_idx ||
+        !packed_logits || !resid || !n_resid)
+        return ORACLE_BAD_ARG;
+    unsigned char *covered = (unsigned char *)calloc((size_t)C, 1);
+    int *seen_in_row = (int *)malloc(sizeof(int) * (size_t)C);
+    oracle_pair *row = (oracle_pair *)malloc(sizeof(oracle_pair) * (size_t)k);
+    if (!covered || !seen_in_row || !row) {
+        free(covered);
+        free(seen_in_row);
+        free(row);
+        return ORACLE_NO_MEMORY;
+    }
+    for (int c = 0; c < C; ++c)
+        seen_in_row[c] = -1;
+    int status = ORACLE_OK;
+    for (int e = 0; e < R && status == ORACLE_OK; ++e) {
+        for (int i = 0; i < k; ++i) {
+            int32_t c = support_idx[(size_t)e * k + i];
+            float v = support_logits[(size_t)e * k + i];
+            if (c < 0 || c >= C || !isfinite(v) || seen_in_row[c] == e) {
+                status = ORACLE_BAD_SUPPORT;
+                break;
+            }
+            seen_in_row[c] = e;
+            row[i].idx = c;
+            row[i].logit = v;
+        }
+        if (status != ORACLE_OK)
+            break;
+        qsort(row, (size_t)k, sizeof(oracle_pair), pair_order);
+        for (int i = 0; i < k; ++i) {
+            packed_idx[(size_t)e * k + i] = row[i].idx;
+            packed_logits[(size_t)e * k + i] = row[i].logit;
+            covered[row[i].idx] = 1;
+        }
+    }
+    if (status == ORACLE_OK) {
+        int m = 0;
+        for (int c = 0; c < C; ++c)
+            if (!covered[c])
+                resid[m++] = c;
+        *n_resid = m;
+    }
+    free(covered);
+    free(seen_in_row);
+    free(row);
+    return status;
+}
+
+/* Sec. 3.3: z = GAP(X), the mean over the H*W positions of each (n, c). */
+void moce_oracle_pool(const float *x, int N, int H, int W, int C, int layout, double *z)
+{
+    int HW = H * W;
+    for (int n = 0; n < N; ++n)
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int p = 0; p < HW; ++p)
+                s += (double)x[x_at(layout, n, p, c, HW, C)];
+            z[(size_t)n * C + c] = s / (double)HW;
+        }
+}
+
+/*
+ * Eq. (tau): tau_e = tau_min + (tau_max - tau_min) * sigma(g(z_{S_e})).
+ * The gate input u is z at the expert's support in deployment order, so u_0
+ * is the descriptor of the expert's most preferred channel (Sec. 3.3).
+ * g(u) = w2 . ReLU(W1 u + b1) + b2, W1 is [k][k] with row j = hidden unit j.
+ * g_out (optional) receives the pre-sigmoid gate value, [N][R].
+ */
+void moce_oracle_gate(const double *z, int N, int C, int R, int k, const int32_t *packed_idx,
+                      const float *W1, const float *b1, const float *w2, float b2,
+                      double tau_min, double tau_max, double *g_out, double *tau)
+{
+    double *u = (double *)malloc(sizeof(double) * (size_t)k);
+    double *h = (double *)malloc(sizeof(double) * (size_t)k);
+    for (int n = 0; n < N; ++n)
+        for (int e = 0; e < R; ++e) {
+            for (int i = 0; i < k; ++i)
+                u[i] = z[(size_t)n * C + packed_idx[(size_t)e * k + i]];
+            for (int j = 0; j < k; ++j) {
+                double s = (double)b1[j];
+                for (int i = 0; i < k; ++i)
+                    s += (double)W1[(size_t)j * k + i] * u[i];
+                h[j] = s > 0.0 ? s : 0.0;
+            }
+            double g = (double)b2;
+            for (int j = 0; j < k; ++j)
+                g += (double)w2[j] * h[j];
+            double sig = 1.0 / (1.0 + exp(-g));
+            if (g_out)
+                g_out[(size_t)n * R + e] = g;
+            tau[(size_t)n * R + e] = tau_min + (tau_max - tau_min) * sig;
+        }
+    free(u);
+    free(h);
+}
+
+/*
+ * Eq. (weights): a_{e,i} = exp(L_{e,i}/tau_e) / sum_j exp(L_{e,j}/tau_e),
+ * evaluated as exp((L_{e,i} - max_j L_{e,j}) / tau_e) / sum (same value).
+ * tau is [N][R], packed_logits [R][k], a is [N][R][k].
+ */
+void moce_oracle_weights(const double *tau, int N, int R, int k, const float *packed_logits,
+                         double *a)
+{
+    for (int n = 0; n < N; ++n)
+        for (int e = 0; e < R; ++e) {
+            const float *L = packed_logits + (size_t)e * k;
+            double t = tau[(size_t)n * R + e];
+            double m = (double)L[0];
+            for (int i = 1; i < k; ++i)
+                if ((double)L[i] > m)
+                    m = (double)L[i];
+            double *ae = a + ((size_t)n * R + e) * k;
+            double s = 0.0;
+            for (int i = 0; i < k; ++i) {
+                ae[i] = exp(((double)L[i] - m) / t);
+                s += ae[i];
+            }
+            for (int i = 0; i < k; ++i)
+                ae[i] /= s;
+        }
+}
+
+/*
+ * Eq. (expert) and Eq. (res): at every position,
+ *   y_e = sum_i a_{e,i} x_{S_e[i]}               for e < R,
+ *   y_R = |U|^-1 sum_{c in U} x_c, or 0 if U is empty.
+ * a is [N][R][k]; y has R + 1 channels in the layout of x.
+ */
+void moce_oracle_mix(const float *x, int N, int H, int W, int C, int layout, int R, int k,
+                     const int32_t *packed_idx, const double *a, const int32_t *resid,
+                     int n_resid, double *y)
+{
+    int HW = H * W;
+    int E = R + 1;
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < HW; ++p) {
+            for (int e = 0; e < R; ++e) {
+                const double *ae = a + ((size_t)n * R + e) * k;
+                double s = 0.0;
+                for (int i = 0; i < k; ++i)
+                    s += ae[i] * (double)x[x_at(layout, n, p, packed_idx[(size_t)e * k + i], HW, C)];
+                y[x_at(layout, n, p, e, HW, E)] = s;
+            }
+            double r = 0.0;
+            if (n_resid > 0) {
+                for (int j = 0; j < n_resid; ++j)
+                    r += (double)x[x_at(layout, n, p, resid[j], HW, C)];
+                r /= (double)n_resid;
+            }
+            y[x_at(layout, n, p, R, HW, E)] = r;
+        }
+}
+
+/*
+ * The whole layer: pool -> gate -> weights -> routed + residual outputs.
+ * Supports must already be packed. z_out [N][C], tau_out [N][R] and
+ * a_out [N][R][k] are optional copies of the intermediates.
+ */
+int moce_oracle_forward(const float *x, int N, int H, int W, int C, int layout, int R, int k,
+                        const int32_t *packed_idx, const float *packed_logits,
+                        const int32_t *resid, int n_resid, const float *W1, const float *b1,
+                        const float *w2, float b2, double tau_min, double tau_max, double *y,
+                        double *z_out, double *tau_out, double *a_out)
+{
+    if (N < 0 || H < 0 || W < 0 || C < 1 || R < 1 || k < 1 || k > C || n_resid < 0 ||
+        n_resid > C || (layout != 0 && layout != 1))
+        return ORACLE_BAD_ARG;
+    double *z = z_out ? z_out : (double *)malloc(sizeof(double) * ((size_t)N * C + 1));
+    double *tau = tau_out ? tau_out : (double *)malloc(sizeof(double) * ((size_t)N * R + 1));
+    double *a = a_out ? a_out : (double *)malloc(sizeof(double) * ((size_t)N * R * k + 1));
+    int status = ORACLE_OK;
+    if (!z || !tau || !a) {
+        status = ORACLE_NO_MEMORY;
+    } else {
+        moce_oracle_pool(x, N, H, W, C, layout, z);
+        moce_oracle_gate(z, N, C, R, k, packed_idx, W1, b1, w2, b2, tau_min, tau_max, NULL, tau);
+        moce_oracle_weights(tau, N, R, k, packed_logits, a);
+        moce_oracle_mix(x, N, H, W, C, layout, R, k, packed_idx, a, resid, n_resid, y);
+    }
+    if (!z_out)
+        free(z);
+    if (!tau_out)
+        free(tau);
+    if (!a_out)
+        free(a);
+    return status;
+}
+
+/*
+ * Brute-force restatement used to pin the oracle above on tiny shapes. It
+ * starts from the full routing matrix L [R][C] (the training-time form,
+ * Sec. 3.2) and shares no step with the functions above:
+ *   - S_e by k rounds of "take the largest remaining logit" (ties: smallest
+ *     channel), not by sorting;
+ *   - U by counting, over all experts, how often each channel is selected;
+ *   - weights as exp(L/tau) / sum exp(L/tau) with no max subtraction;
+ *   - the layer as a dense matrix W_eff [R+1][C] per example, applied to the
+ *     channel vector of every position with a plain triple loop.
+ * Used only with small logits, where exp(L/tau) cannot overflow.
+ */
+int moce_oracle_bruteforce_forward(const float *x, int N, int H, int W, int C, int layout, int R,
+                                   int k, const float *L, const float *W1, const float *b1,
+                                   const float *w2, float b2, double tau_min, double tau_max,
+                                   double *y)
+{
+    if (N < 0 || H < 0 || W < 0 || C < 1 || R < 1 || k < 1 || k > C || (layout != 0 && layout != 1))
+        return ORACLE_BAD_ARG;
+    int HW = H * W;
+    int E = R + 1;
+    int *sel = (int *)malloc(sizeof(int) * (size_t)R * k);
+    int *count = (int *)calloc((size_t)C, sizeof(int));
+    unsigned char *taken = (unsigned char *)malloc((size_t)C);
+    double *Weff = (double *)malloc(sizeof(double) * (size_t)E * C);
+    double *zn = (double *)malloc(sizeof(double) * (size_t)C);
+    double *hid = (double *)malloc(sizeof(double) * (size_t)k);
+    if (!sel || !count || !taken || !Weff || !zn || !hid) {
+        free(sel); free(count); free(taken); free(Weff); free(zn); free(hid);
+        return ORACLE_NO_MEMORY;
+    }
+    for (int e = 0; e < R; ++e) {
+        memset(taken, 0, (size_t)C);
+        for (int r = 0; r < k; ++r) {
+            int best = -1;
+            for (int c = 0; c < C; ++c) {
+                if (taken[c])
+                    continue;
+                if (best < 0 || L[(size_t)e * C + c] > L[(size_t)e * C + best])
+                    best = c;
+            }
+            taken[best] = 1;
+            sel[(size_t)e * k + r] = best;
+            count[best] += 1;
+        }
+    }
+    int nU = 0;
+    for (int c = 0; c < C; ++c)
+        nU += (count[c] == 0);
+    for (int n = 0; n < N; ++n) {
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int p = 0; p < HW; ++p)
+                s += (double)x[x_at(layout, n, p, c, HW, C)];
+            zn[c] = s / (double)HW;
+        }
+        for (size_t q = 0; q < (size_t)E * C; ++q)
+            Weff[q] = 0.0;
+        for (int e = 0; e < R; ++e) {
+            /* gate: input position r is the r-th selected (r-th largest) channel */
+            double g = (double)b2;
+            for (int j = 0; j < k; ++j) {
+                double s = (double)b1[j];
+                for (int r = 0; r < k; ++r)
+                    s += (double)W1[(size_t)j * k + r] * zn[sel[(size_t)e * k + r]];
+                if (s > 0.0)
+                    g += (double)w2[j] * s;
+            }
+            double t = tau_min + (tau_max - tau_min) / (1.0 + exp(-g));
+            double den = 0.0;
+            for (int r = 0; r < k; ++r)
+                den += exp((double)L[(size_t)e * C + sel[(size_t)e * k + r]] / t);
+            for (int r = 0; r < k; ++r) {
+                int c = sel[(size_t)e * k + r];
+                Weff[(size_t)e * C + c] += exp((double)L[(size_t)e * C + c] / t) / den;
+            }
+        }
+        if (nU > 0)
+            for (int c = 0; c < C; ++c)
+                if (count[c] == 0)
+                    Weff[(size_t)R * C + c] = 1.0 / (double)nU;
+        for (int p = 0; p < HW; ++p)
+            for (int o = 0; o < E; ++o) {
+                double s = 0.0;
+                for (int c = 0; c < C; ++c)
+                    s += Weff[(size_t)o * C + c] * (double)x[x_at(layout, n, p, c, HW, C)];
+                y[x_at(layout, n, p, o, HW, E)] = s;
+            }
+    }
+    free(sel); free(count); free(taken); free(Weff); free(zn); free(hid);
+    return ORACLE_OK;
+}

@@ -1,0 +1,87 @@
+"""Each planted mistake in a copy of the oracle must be caught by the pins.
+
+The mutants are textual edits of oracle/moce_oracle.c compiled to a temporary
+library; the real oracle is never modified.
+"""
+import os
+import subprocess
+
+import pytest
+
+import oracle
+import test_oracle_pins as pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "moce_oracle.c")
+
+MUTANTS = {
+    "softmax_sign": ("ae[i] = exp(((double)L[i] - m) / t);", "ae[i] = exp((m - (double)L[i]) / t);"),
+    "gate_input_reversed": ("u[i] = z[(size_t)n * C + packed_idx[(size_t)e * k + i]];",
+                            "u[i] = z[(size_t)n * C + packed_idx[(size_t)e * k + (k - 1 - i)]];"),
+    "gate_W1_transposed": ("s += (double)W1[(size_t)j * k + i] * u[i];",
+                           "s += (double)W1[(size_t)i * k + j] * u[i];"),
+    "gate_b1_dropped": ("double s = (double)b1[j];\n                for (int i = 0;",
+                        "double s = 0.0;\n                for (int i = 0;"),
+    "gate_relu_dropped": ("h[j] = s > 0.0 ? s : 0.0;", "h[j] = s;"),
+    "gate_b2_dropped": ("double g = (double)b2;\n            for (int j = 0; j < k; ++j)\n                g += (double)w2[j] * h[j];",
+                        "double g = 0.0;\n            for (int j = 0; j < k; ++j)\n                g += (double)w2[j] * h[j];"),
+    "sigmoid_sign": ("double sig = 1.0 / (1.0 + exp(-g));", "double sig = 1.0 / (1.0 + exp(g));"),
+    "tau_reversed": ("tau[(size_t)n * R + e] = tau_min + (tau_max - tau_min) * sig;",
+                     "tau[(size_t)n * R + e] = tau_max - (tau_max - tau_min) * sig;"),
+    "pool_not_divided": ("z[(size_t)n * C + c] = s / (double)HW;", "z[(size_t)n * C + c] = s;"),
+    "mix_index_shift": ("s += ae[i] * (double)x[x_at(layout, n, p, packed_idx[(size_t)e * k + i], HW, C)];",
+                        "s += ae[i] * (double)x[x_at(layout, n, p, packed_idx[(size_t)e * k + (i + 1) % k], HW, C)];"),
+    "mix_last_term_dropped": ("for (int i = 0; i < k; ++i)\n                    s += ae[i]",
+                              "for (int i = 0; i < k - 1; ++i)\n                    s += ae[i]"),
+    "residual_not_divided": ("r /= (double)n_resid;", "r *= 1.0;"),
+    "residual_complement_flipped": ("if (!covered[c])\n                resid[m++] = c;",
+                                    "if (covered[c])\n                resid[m++] = c;"),
+    "pack_ascending": ("if (a->logit > b->logit)\n        return -1;", "if (a->logit < b->logit)\n        return -1;"),
+    "pack_ties_descending_index": ("return (a->idx > b->idx) - (a->idx < b->idx);",
+                                   "return (a->idx < b->idx) - (a->idx > b->idx);"),
+    "pack_no_duplicate_check": ("seen_in_row[c] == e", "0"),
+}
+
+PIN_CHECKS = [
+    pins.test_worked_tiny_layer,
+    lambda: pins.test_pack_equals_bruteforce_sort(0),
+    pins.test_pack_permutation_invariant,
+    pins.test_pack_ties_and_signed_zero,
+    lambda: pins.test_pack_rejects("dup"),
+    lambda: pins.test_cyclic_supports_residual_closed_form(64, 15, 4),
+    lambda: pins.test_pool_closed_forms("nhwc"),
+    pins.test_gate_zero_hidden_gives_sigmoid_of_bias,
+    pins.test_gate_reads_inputs_in_descending_logit_order_and_w1_rows_are_hidden_units,
+    pins.test_gate_relu_clamps,
+    pins.test_weights_convex_and_order_invariant,
+    pins.test_weights_unit_temperature_is_plain_softmax,
+    pins.test_weights_temperature_limits,
+    pins.test_mix_bounds_and_residual_mean,
+    pins.test_empty_residual_is_exactly_zero,
+    lambda: pins.test_forward_equals_bruteforce("nhwc", 0),
+    pins.test_fixed_temperature_is_a_linear_map,
+]
+
+
+def _build_mutant(tmp_path, name, old, new):
+    text = open(SRC).read()
+    assert text.count(old) == 1, f"mutation site for {name} not unique"
+    src = tmp_path / f"{name}.c"
+    src.write_text(text.replace(old, new))
+    so = tmp_path / f"lib{name}.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-o", str(so), str(src), "-lm"],
+                   check=True)
+    return str(so)
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_reject_mutant(tmp_path, name):
+    old, new = MUTANTS[name]
+    so = _build_mutant(tmp_path, name, old, new)
+    failures = 0
+    with oracle._use_library(so):
+        for check in PIN_CHECKS:
+            try:
+                check()
+            except (Exception, pytest.fail.Exception):  # a failed assertion or an oracle error
+                failures += 1
+    assert failures > 0, f"no pin catches mutant {name}"

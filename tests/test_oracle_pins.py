@@ -1,0 +1,308 @@
+"""Pins of the CPU oracle to facts fixed by the paper and by mathematics.
+
+None of these re-types the oracle's own formulas: each checks a worked
+example, a closed form, an invariant the paper states, a special case that
+reduces to a library routine, or a brute-force restatement on tiny inputs.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.special import softmax as sp_softmax
+
+import oracle
+from paper_2608_23794_gb300 import synth
+
+GOLD_DIR = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rand_supports(rng, C, R, k):
+    idx = np.stack([rng.choice(C, size=k, replace=False) for _ in range(R)]).astype(np.int32)
+    lg = rng.standard_normal((R, k)).astype(np.float32)
+    return idx, lg
+
+
+# ---------------------------------------------------------------- worked example
+
+
+def test_worked_tiny_layer():
+    g = json.load(open(os.path.join(GOLD_DIR, "worked_tiny_layer.json")))
+    x = np.array(g["x_nhwc"], np.float32)
+    pidx, plog, resid = oracle.pack(np.array(g["support_idx"]), np.array(g["support_logits"]), g["C"])
+    ex = g["expected"]
+    assert pidx.tolist() == ex["packed_idx"]
+    assert resid.tolist() == ex["resid"]
+    y, z, tau, a = oracle.forward(x, "nhwc", pidx, plog, resid, np.array(g["W1"]), np.array(g["b1"]),
+                                  np.array(g["w2"]), g["b2"], g["tau_min"], g["tau_max"],
+                                  intermediates=True)
+    tol = g["rel_tol"]
+    np.testing.assert_allclose(z, ex["z"], rtol=tol)
+    np.testing.assert_allclose(tau, ex["tau"], rtol=tol)
+    np.testing.assert_allclose(a, ex["a"], rtol=tol)
+    np.testing.assert_allclose(y, ex["y_nhwc"], rtol=tol)
+
+
+# ---------------------------------------------------------------- packing
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_pack_equals_bruteforce_sort(seed):
+    rng = np.random.default_rng(seed)
+    C, R, k = 37, 9, 5
+    idx, lg = _rand_supports(rng, C, R, k)
+    lg[:, 1] = lg[:, 0]  # force ties in every row
+    pidx, plog, resid = oracle.pack(idx, lg, C)
+    for e in range(R):
+        want = sorted(zip(idx[e].tolist(), lg[e].tolist()), key=lambda t: (-t[1], t[0]))
+        assert pidx[e].tolist() == [t[0] for t in want]
+        assert plog[e].tolist() == [t[1] for t in want]
+    assert resid.tolist() == sorted(set(range(C)) - set(idx.ravel().tolist()))
+
+
+def test_pack_permutation_invariant():
+    rng = np.random.default_rng(3)
+    C, R, k = 64, 12, 7
+    idx, lg = _rand_supports(rng, C, R, k)
+    ref = oracle.pack(idx, lg, C)
+    for _ in range(4):
+        perm = np.stack([rng.permutation(k) for _ in range(R)])
+        got = oracle.pack(np.take_along_axis(idx, perm, 1), np.take_along_axis(lg, perm, 1), C)
+        for a, b in zip(ref, got):
+            assert a.tobytes() == b.tobytes()
+
+
+def test_pack_ties_and_signed_zero():
+    idx = np.array([[5, 2, 9, 0]], np.int32)
+    lg = np.array([[0.0, -0.0, 1.5, 0.0]], np.float32)
+    pidx, plog, _ = oracle.pack(idx, lg, 10)
+    assert pidx.tolist() == [[9, 0, 2, 5]]
+
+
+@pytest.mark.parametrize("bad", ["range_hi", "range_lo", "dup", "nan", "inf"])
+def test_pack_rejects(bad):
+    idx = np.array([[0, 1, 2], [3, 4, 5]], np.int32)
+    lg = np.zeros((2, 3), np.float32)
+    if bad == "range_hi":
+        idx[1, 2] = 6
+    elif bad == "range_lo":
+        idx[0, 0] = -1
+    elif bad == "dup":
+        idx[1, 2] = 3
+    elif bad == "nan":
+        lg[0, 1] = np.nan
+    else:
+        lg[1, 0] = np.inf
+    with pytest.raises(oracle.OracleError) as ei:
+        oracle.pack(idx, lg, 6)
+    assert ei.value.status == oracle.BAD_SUPPORT
+
+
+@pytest.mark.parametrize("C,R,k", [(64, 16, 4), (64, 15, 4), (30, 4, 7), (256, 64, 16)])
+def test_cyclic_supports_residual_closed_form(C, R, k):
+    # Sec. 4.5 cyclic supports: experts cover channels 0 .. R*k-1 (mod C), so
+    # U = {R*k, ..., C-1} when R*k < C and U is empty otherwise.
+    idx = synth.cyclic_supports(C, R, k)
+    lg = np.random.default_rng(0).standard_normal((R, k)).astype(np.float32)
+    _, _, resid = oracle.pack(idx, lg, C)
+    want = list(range(R * k, C)) if R * k < C else []
+    assert resid.tolist() == want
+
+
+def test_topk_equals_stable_argsort():
+    rng = np.random.default_rng(11)
+    L = rng.standard_normal((7, 40)).astype(np.float32)
+    L[:, 5] = L[:, 6]  # ties
+    idx, lg = oracle.topk(L, 9)
+    ref = np.argsort(-L, axis=1, kind="stable")[:, :9]
+    assert idx.tolist() == ref.tolist()
+    assert lg.tolist() == np.take_along_axis(L, ref, 1).tolist()
+
+
+# ---------------------------------------------------------------- pooling
+
+
+@pytest.mark.parametrize("layout", ["nhwc", "nchw"])
+def test_pool_closed_forms(layout):
+    N, H, W, C = 2, 5, 3, 4
+    const = np.full((N, H, W, C), 0.75, np.float32)
+    ramp = np.broadcast_to(np.arange(H * W, dtype=np.float32).reshape(1, H, W, 1), (N, H, W, C))
+    for x, want in ((const, 0.75), (ramp, (H * W - 1) / 2.0)):
+        z = oracle.pool(synth.x_to_layout(np.ascontiguousarray(x), "nhwc", layout), layout)
+        assert np.all(z == want)
+    rnd = np.random.default_rng(0).standard_normal((N, H, W, C)).astype(np.float32)
+    z = oracle.pool(synth.x_to_layout(rnd, "nhwc", layout), layout)
+    np.testing.assert_allclose(z, rnd.astype(np.float64).mean(axis=(1, 2)), rtol=1e-12, atol=1e-15)
+
+
+# ---------------------------------------------------------------- gate
+
+
+def test_gate_zero_hidden_gives_sigmoid_of_bias():
+    # W1 = 0, b1 = 0 -> h = 0 -> g = b2; sigma(0) = 1/2, sigma(ln 3) = 3/4.
+    k, R, C = 3, 4, 10
+    pidx = np.array([[0, 1, 2]] * R, np.int32)
+    z = np.random.default_rng(1).standard_normal((2, C))
+    zeros = np.zeros((k, k), np.float32)
+    for b2, sig in ((0.0, 0.5), (math.log(3.0), 0.75)):
+        tau = oracle.gate(z, pidx, zeros, np.zeros(k), np.ones(k), b2, 0.2, 6.0)
+        np.testing.assert_allclose(tau, 0.2 + 5.8 * sig, rtol=1e-7)
+
+
+def test_gate_reads_inputs_in_descending_logit_order_and_w1_rows_are_hidden_units():
+    # W1 = E_01 (hidden unit 0 reads input position 1), w2 = e_0: g = ReLU(u_1),
+    # the descriptor of each expert's SECOND most preferred channel.
+    rng = np.random.default_rng(7)
+    C, R, k = 12, 5, 3
+    idx, lg = _rand_supports(rng, C, R, k)
+    pidx, plog, _ = oracle.pack(idx, lg, C)
+    z = rng.uniform(0.5, 2.0, size=(2, C))
+    W1 = np.zeros((k, k), np.float32)
+    W1[0, 1] = 1.0
+    w2 = np.zeros(k, np.float32)
+    w2[0] = 1.0
+    _, g = oracle.gate(z, pidx, W1, np.zeros(k), w2, 0.0, 0.2, 6.0, return_g=True)
+    for n in range(2):
+        for e in range(R):
+            second = idx[e][np.argsort(-lg[e], kind="stable")[1]]
+            assert g[n, e] == pytest.approx(z[n, second], rel=1e-12)
+
+
+def test_gate_relu_clamps():
+    C, R, k = 4, 1, 2
+    pidx = np.array([[0, 1]], np.int32)
+    z = np.array([[-3.0, 2.0, 0.0, 0.0]])
+    W1 = np.eye(2, dtype=np.float32)
+    _, g = oracle.gate(z, pidx, W1, np.zeros(2), np.ones(2), 0.5, 0.2, 6.0, return_g=True)
+    # h = ReLU([-3, 2]) = [0, 2]; g = 0 + 2 + 0.5
+    assert g[0, 0] == pytest.approx(2.5, rel=1e-15)
+
+
+def test_gate_range():
+    cfg = synth.CONFIGS["tiny_f32_nchw"]
+    lay = synth.make_layer(cfg, 5)
+    pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, cfg.C_in)
+    z = oracle.pool(lay.x, cfg.layout) * 50.0
+    tau = oracle.gate(z, pidx, lay.W1 * 10, lay.b1, lay.w2 * 10, float(lay.b2[0]), 0.2, 6.0)
+    assert np.all(tau >= 0.2) and np.all(tau <= 6.0)
+
+
+# ---------------------------------------------------------------- weights
+
+
+def _weights_setup(seed=0, R=6, k=8):
+    rng = np.random.default_rng(seed)
+    idx, lg = _rand_supports(rng, 64, R, k)
+    return oracle.pack(idx, lg, 64)
+
+
+def test_weights_convex_and_order_invariant():
+    pidx, plog, _ = _weights_setup()
+    tau = np.random.default_rng(1).uniform(0.2, 6.0, size=(3, plog.shape[0]))
+    a = oracle.weights(tau, plog)
+    np.testing.assert_allclose(a.sum(-1), 1.0, rtol=1e-14)
+    assert np.all(a > 0)
+    # Sec. 3.3: along the temperature curve the ordering of the weights never changes;
+    # positions are in descending-logit order, so a is non-increasing.
+    assert np.all(np.diff(a, axis=-1) <= 1e-15)
+
+
+def test_weights_unit_temperature_is_plain_softmax():
+    pidx, plog, _ = _weights_setup(2)
+    tau = np.ones((2, plog.shape[0]))
+    a = oracle.weights(tau, plog)
+    np.testing.assert_allclose(a[0], sp_softmax(plog.astype(np.float64), axis=-1), rtol=1e-13)
+
+
+def test_weights_temperature_limits():
+    pidx, plog, _ = _weights_setup(4)
+    R, k = plog.shape
+    a_hot = oracle.weights(np.full((1, R), 1e4), plog)
+    spread = float(plog.max() - plog.min())
+    assert np.max(np.abs(a_hot - 1.0 / k)) < 2 * spread / 1e4
+    gaps = plog[:, 0] - plog[:, 1]
+    a_cold = oracle.weights(np.full((1, R), 1e-3), plog)
+    for e in range(R):
+        if gaps[e] >= 0.05:
+            assert a_cold[0, e, 0] == 1.0 and np.all(a_cold[0, e, 1:] < 1e-20)
+
+
+# ---------------------------------------------------------------- mixing + residual
+
+
+def test_mix_bounds_and_residual_mean():
+    cfg = synth.CONFIGS["tiny_f32_nchw"]
+    lay = synth.make_layer(cfg, 1)
+    pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, cfg.C_in)
+    y = oracle.forward(lay.x, "nchw", pidx, plog, resid, lay.W1, lay.b1, lay.w2, float(lay.b2[0]),
+                       0.2, 6.0)
+    x = lay.x.astype(np.float64)
+    for e in range(cfg.C_out):
+        xs = x[:, pidx[e]]  # [N, k, H, W]
+        assert np.all(y[:, e] >= xs.min(axis=1) - 1e-12)
+        assert np.all(y[:, e] <= xs.max(axis=1) + 1e-12)
+    assert len(resid) >= cfg.C_in - cfg.support_pool
+    np.testing.assert_allclose(y[:, cfg.C_out], x[:, resid].mean(axis=1), rtol=1e-13)
+
+
+def test_empty_residual_is_exactly_zero():
+    C, R, k = 8, 4, 2  # cyclic supports cover all 8 channels
+    idx = synth.cyclic_supports(C, R, k)
+    lg = np.random.default_rng(0).standard_normal((R, k)).astype(np.float32)
+    pidx, plog, resid = oracle.pack(idx, lg, C)
+    assert resid.size == 0
+    x = np.random.default_rng(1).uniform(1, 2, size=(2, 3, 3, C)).astype(np.float32)
+    y = oracle.forward(x, "nhwc", pidx, plog, resid, np.zeros((k, k)), np.zeros(k), np.zeros(k),
+                       0.0, 0.2, 6.0)
+    assert np.all(y[..., R] == 0.0)
+
+
+@pytest.mark.parametrize("layout", ["nhwc", "nchw"])
+@pytest.mark.parametrize("seed", range(3))
+def test_forward_equals_bruteforce(layout, seed):
+    rng = np.random.default_rng(100 + seed)
+    N, H, W, C, R, k = 2, 3, 4, 11, 5, 3
+    L = rng.standard_normal((R, C)).astype(np.float32)
+    L[:, 2] = L[:, 3]
+    x = rng.standard_normal((N, H, W, C)).astype(np.float32)
+    x = synth.x_to_layout(x, "nhwc", layout)
+    W1 = rng.standard_normal((k, k)).astype(np.float32)
+    b1 = rng.standard_normal(k).astype(np.float32)
+    w2 = rng.standard_normal(k).astype(np.float32)
+    b2 = float(rng.standard_normal())
+    sidx, slog = oracle.topk(L, k)
+    perm = np.stack([rng.permutation(k) for _ in range(R)])
+    pidx, plog, resid = oracle.pack(np.take_along_axis(sidx, perm, 1),
+                                    np.take_along_axis(slog, perm, 1), C)
+    y = oracle.forward(x, layout, pidx, plog, resid, W1, b1, w2, b2, 0.2, 6.0)
+    yb = oracle.bruteforce_forward(x, layout, L, k, W1, b1, w2, b2, 0.2, 6.0)
+    np.testing.assert_allclose(y, yb, rtol=1e-12, atol=1e-13)
+
+
+def test_fixed_temperature_is_a_linear_map():
+    # tau_min = tau_max = T: the layer is y = W_eff x with W_eff built from
+    # scipy's softmax of L/T on the support and 1/|U| on U; applied with einsum.
+    rng = np.random.default_rng(9)
+    N, H, W, C, R, k, T = 2, 4, 5, 16, 6, 4, 0.7
+    idx, lg = _rand_supports(rng, 12, R, k)  # channels 12..15 stay in U
+    x = rng.standard_normal((N, H, W, C)).astype(np.float32)
+    pidx, plog, resid = oracle.pack(idx, lg, C)
+    y = oracle.forward(x, "nhwc", pidx, plog, resid, rng.standard_normal((k, k)),
+                       rng.standard_normal(k), rng.standard_normal(k), 0.3, T, T)
+    Weff = np.zeros((R + 1, C))
+    for e in range(R):
+        Weff[e, idx[e]] = sp_softmax(lg[e].astype(np.float64) / T)
+    Weff[R, resid] = 1.0 / len(resid)
+    ref = np.einsum("oc,nhwc->nhwo", Weff, x.astype(np.float64))
+    np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-13)
+
+
+def test_layouts_agree():
+    cfg = synth.CONFIGS["tiny_f32_nchw"]
+    lay = synth.make_layer(cfg, 2)
+    pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, cfg.C_in)
+    args = (pidx, plog, resid, lay.W1, lay.b1, lay.w2, float(lay.b2[0]), 0.2, 6.0)
+    y_nchw = oracle.forward(lay.x, "nchw", *args)
+    y_nhwc = oracle.forward(synth.x_to_layout(lay.x, "nchw", "nhwc"), "nhwc", *args)
+    assert np.array_equal(synth.x_to_layout(y_nhwc, "nhwc", "nchw"), y_nchw)
