@@ -1,0 +1,184 @@
+/*
+ * moce.h - C ABI of the MoCE layer forward on NVIDIA GB300 (sm_103a).
+ *
+ * A Mixture of Channel Experts layer ("Mixture of Channel Experts: Static
+ * Sparse Supports with Input-Adaptive Mixing for Pointwise Projections",
+ * Sec. 3) replaces a dense 1x1 projection C_in -> C_out + 1. Each of the
+ * C_out routed experts mixes k channels of a static support with
+ * softmax weights whose temperature is predicted per example from the pooled
+ * descriptors of that support; one residual expert averages the channels no
+ * routed expert selects.
+ *
+ *   z        = GAP(x)                                            Sec. 3.3
+ *   tau[n,e] = tau_min + (tau_max - tau_min) * sigma(g(z[n, S_e]))  Eq. (tau)
+ *              g(u) = w2 . ReLU(W1 u + b1) + b2, u in descending-logit order
+ *              (Sec. 3.3 ordering rule; gate shape of Sec. 4.1)
+ *   a[n,e,i] = softmax_i(L[e,i] / tau[n,e])                     Eq. (weights)
+ *   y[n,p,e] = sum_i a[n,e,i] x[n,p,S_e[i]]        e < C_out    Eq. (expert)
+ *   y[n,p,C_out] = mean_{c in U} x[n,p,c], 0 if U is empty      Eq. (res)
+ *
+ * Conventions shared by every entry point:
+ *   - All tensor pointers are DEVICE pointers unless the name ends in _host.
+ *     The caller owns every buffer; the library never allocates memory and
+ *     keeps no global state.
+ *   - Calls are asynchronous on `stream` unless stated otherwise. A NULL
+ *     stream is the legacy default stream.
+ *   - Arguments are validated on the host before any launch; an invalid
+ *     argument returns MOCE_ERR_INVALID_VALUE and enqueues nothing. A failed
+ *     launch returns MOCE_ERR_CUDA. No call traps or asserts on the device.
+ *   - Shapes: N examples (0..65535), H x W positions, C_in input channels (1..65535, the
+ *     16-bit index range of the deployment format, Sec. 3.5), C_out routed
+ *     experts (>= 1), support size k (1..C_in).
+ *   - x layout MOCE_NHWC: x[((n*H + h)*W + w)*C_in + c]; MOCE_NCHW:
+ *     x[((n*C_in + c)*H + h)*W + w]. y has C_out + 1 channels in the same
+ *     layout and dtype as x, the residual expert at channel C_out.
+ *   - dtype MOCE_BF16 stores bfloat16 bit patterns; all arithmetic is fp32 and
+ *     outputs are rounded to nearest even.
+ */
+#ifndef MOCE_H
+#define MOCE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum moce_status {
+    MOCE_OK = 0,
+    MOCE_ERR_INVALID_VALUE = 1, /* bad shape, null pointer, misaligned buffer, small workspace */
+    MOCE_ERR_BAD_SUPPORT = 2,   /* support index out of range / repeated in a row, or non-finite logit */
+    MOCE_ERR_UNSUPPORTED = 3,   /* valid arguments this build has no kernel for */
+    MOCE_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
+    MOCE_ERR_TIMEOUT = 5        /* a bounded device-side wait ran out (see moce_check_device_error) */
+} moce_status_t;
+
+typedef enum moce_dtype { MOCE_F32 = 0, MOCE_BF16 = 1 } moce_dtype_t;
+typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
+
+/* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */
+typedef struct CUstream_st *moce_stream_t;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *moce_status_string(moce_status_t status);
+
+/*
+ * Bytes of device workspace moce_pack_supports needs (coverage bitmap, error
+ * word, |U| counter). Returns 0 for invalid shapes.
+ */
+size_t moce_pack_workspace_bytes(int C_in, int C_out, int k);
+
+/*
+ * Deployment packing of static supports (Sec. 3.2: supports are fixed at
+ * inference; Sec. 3.5 "Storage": deployment keeps the selected logits and
+ * their indices; Sec. 3.3: the gate input is ordered by descending routing
+ * logit; Sec. 3.4: U = channels no expert selects).
+ *
+ *   support_idx     [C_out*k] int32, row e = the k channels of expert e, any order
+ *   support_logits  [C_out*k] fp32, the routing logit of each selected channel
+ *   packed_idx      [C_out*k] int32 out: each row sorted by logit descending,
+ *                   equal logits by ascending channel (-0.0 equals +0.0)
+ *   packed_logits   [C_out*k] fp32 out: the logits in the same order
+ *   resid_idx       [C_in] int32 out: U in ascending order, first *n_resid_host valid
+ *   n_resid_host    HOST int32 out: |U|
+ *   ws, ws_bytes    device workspace, >= moce_pack_workspace_bytes(C_in, C_out, k),
+ *                   no alignment beyond 4 bytes, contents need not be initialised
+ *
+ * SYNCHRONOUS: returns after the result is complete (it synchronises
+ * `stream`). Rejects an index outside [0, C_in), an index repeated within one
+ * expert, or a NaN/Inf logit with MOCE_ERR_BAD_SUPPORT; outputs are then
+ * unspecified. Inputs and outputs must not overlap. Output is bit-exact and
+ * independent of the input row order.
+ */
+moce_status_t moce_pack_supports(int C_in, int C_out, int k, const int32_t *support_idx,
+                                 const float *support_logits, int32_t *packed_idx,
+                                 float *packed_logits, int32_t *resid_idx, int32_t *n_resid_host,
+                                 void *ws, size_t ws_bytes, moce_stream_t stream);
+
+/*
+ * Bytes of device workspace that moce_pool and moce_forward need for a layer
+ * of this shape (pooling partials, z, tau, mixing weights, scheduler
+ * control words). Returns 0 for invalid shapes.
+ */
+size_t moce_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k);
+
+/*
+ * Zero-fill a workspace (cudaMemsetAsync on `stream`). moce_forward requires
+ * a workspace that was zero-filled before its first use (this call, or any
+ * zero fill); each forward leaves its scheduler words ready for the next one.
+ * Call it again after a forward reported MOCE_ERR_TIMEOUT.
+ */
+moce_status_t moce_workspace_init(void *ws, size_t ws_bytes, moce_stream_t stream);
+
+/*
+ * Byte offsets inside the forward workspace where the last moce_forward left
+ * z [N*C_in] fp32 and tau [N*C_out] fp32 (for inspection and tests).
+ */
+moce_status_t moce_workspace_offsets(int N, int H, int W, int C_in, int C_out, int k,
+                                     size_t *z_offset, size_t *tau_offset);
+
+/*
+ * Global average pooling (Sec. 3.3): z[n*C_in + c] = mean over the H*W
+ * positions of x[n, :, :, c], fp32 accumulation in a fixed order
+ * (deterministic). x: device, layout/dtype as given; NHWC with bf16 needs
+ * C_in % 8 == 0 and a 16-byte aligned x for the vector path, otherwise a
+ * scalar path runs. z: device fp32 [N*C_in]. ws >= moce_workspace_bytes.
+ * H*W must be >= 1.
+ */
+moce_status_t moce_pool(const void *x, int N, int H, int W, int C_in, moce_dtype_t dtype,
+                        moce_layout_t layout, float *z, void *ws, size_t ws_bytes,
+                        moce_stream_t stream);
+
+/*
+ * Temperature gate and mixing weights (Eq. (tau), Eq. (weights); gate shape
+ * of Sec. 4.1).
+ *   z               [N*C_in] fp32 pooled descriptors
+ *   packed_idx      [C_out*k] int32, packed_logits [C_out*k] fp32: from
+ *                   moce_pack_supports (position 0 holds the largest logit)
+ *   W1 [k*k] fp32 row-major, W1[j*k + i] = weight from gate input i to hidden
+ *   unit j; b1 [k]; w2 [k]; b2 [1]: all device fp32
+ *   tau_min <= tau_max, tau_min > 0, both finite
+ *   tau             [N*C_out] fp32 out
+ *   mix_w           [N*C_out*k] fp32 out, or NULL to skip the weights
+ */
+moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
+                        const int32_t *packed_idx, const float *packed_logits, const float *W1,
+                        const float *b1, const float *w2, const float *b2, float tau_min,
+                        float tau_max, float *tau, float *mix_w, moce_stream_t stream);
+
+/*
+ * The whole layer forward (Sec. 3.3-3.4): pooling, gate, weights, routed
+ * mixing and residual, y with C_out + 1 channels in x's layout and dtype.
+ *   packed_idx/packed_logits/resid_idx/n_resid: from moce_pack_supports
+ *   (0 <= n_resid <= C_in; resid_idx may be NULL when n_resid == 0)
+ *   gate parameters and tau bounds as in moce_gate
+ *   y: device, must not overlap x
+ *   ws, ws_bytes: >= moce_workspace_bytes(N, H, W, C_in, C_out, k), 256-byte
+ *   aligned, zero-filled before its first use (moce_workspace_init); one
+ *   workspace serves one stream at a time.
+ * NHWC bf16 with C_in % 8 == 0 and 16-byte aligned x runs one fused
+ * persistent kernel; other layouts/dtypes run a sequence of kernels.
+ * Asynchronous; device-side failures of the fused kernel (a bounded wait
+ * that ran out) are reported by moce_check_device_error.
+ */
+moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                           moce_dtype_t dtype, moce_layout_t layout, const int32_t *packed_idx,
+                           const float *packed_logits, const int32_t *resid_idx, int n_resid,
+                           const float *W1, const float *b1, const float *w2, const float *b2,
+                           float tau_min, float tau_max, void *y, void *ws, size_t ws_bytes,
+                           moce_stream_t stream);
+
+/*
+ * SYNCHRONOUS: waits for `stream`, then reads the device error word the
+ * forward kernels leave in `ws` (a forward workspace). Returns MOCE_OK,
+ * MOCE_ERR_TIMEOUT (a bounded inter-CTA wait gave up; outputs of that call
+ * are invalid and the workspace must be re-initialised) or MOCE_ERR_CUDA.
+ */
+moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOCE_H */

@@ -1,0 +1,181 @@
+// Host entry points of the C ABI declared in include/moce.h: argument
+// validation, workspace layout and kernel selection. Every check happens on
+// the host before anything is enqueued.
+#include <math.h>
+
+#include "moce_internal.cuh"
+
+using namespace moce;
+
+namespace {
+
+constexpr int kMaxChannels = 65535;  // 16-bit support indices (Sec. 3.5)
+
+bool shape_ok(int N, int H, int W, int C, int R, int k) {
+    if (N < 0 || N > 65535 || H < 0 || W < 0) return false;  // N is a grid dimension
+    if (C < 1 || C > kMaxChannels || R < 1 || k < 1 || k > C) return false;
+    if ((long long)H * W > (1ll << 30)) return false;
+    if ((long long)N * H * W * (C > R + 1 ? C : R + 1) > (1ll << 46)) return false;
+    if ((long long)R * k > (1ll << 31) - 1) return false;
+    return true;
+}
+
+bool dtype_ok(moce_dtype_t d) { return d == MOCE_F32 || d == MOCE_BF16; }
+bool layout_ok(moce_layout_t l) { return l == MOCE_NHWC || l == MOCE_NCHW; }
+
+bool tau_ok(float tmin, float tmax) {
+    return isfinite(tmin) && isfinite(tmax) && tmin > 0.f && tmin <= tmax;
+}
+
+moce_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? MOCE_OK : MOCE_ERR_CUDA; }
+
+size_t pack_ws_bytes(int C) { return (2 + (size_t)(C + 31) / 32) * 4; }
+
+}  // namespace
+
+namespace moce {
+size_t gate_smem_bytes(int k);
+}
+
+extern "C" {
+
+const char *moce_status_string(moce_status_t s) {
+    switch (s) {
+    case MOCE_OK: return "MOCE_OK";
+    case MOCE_ERR_INVALID_VALUE: return "MOCE_ERR_INVALID_VALUE";
+    case MOCE_ERR_BAD_SUPPORT: return "MOCE_ERR_BAD_SUPPORT";
+    case MOCE_ERR_UNSUPPORTED: return "MOCE_ERR_UNSUPPORTED";
+    case MOCE_ERR_CUDA: return "MOCE_ERR_CUDA";
+    case MOCE_ERR_TIMEOUT: return "MOCE_ERR_TIMEOUT";
+    }
+    return "MOCE_ERR_UNKNOWN";
+}
+
+size_t moce_pack_workspace_bytes(int C_in, int C_out, int k) {
+    if (!shape_ok(0, 0, 0, C_in, C_out, k)) return 0;
+    return pack_ws_bytes(C_in);
+}
+
+moce_status_t moce_pack_supports(int C_in, int C_out, int k, const int32_t *support_idx,
+                                 const float *support_logits, int32_t *packed_idx,
+                                 float *packed_logits, int32_t *resid_idx, int32_t *n_resid_host,
+                                 void *ws, size_t ws_bytes, moce_stream_t stream) {
+    if (!shape_ok(0, 0, 0, C_in, C_out, k)) return MOCE_ERR_INVALID_VALUE;
+    if (!support_idx || !support_logits || !packed_idx || !packed_logits || !resid_idx ||
+        !n_resid_host || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    if (ws_bytes < pack_ws_bytes(C_in) || (reinterpret_cast<uintptr_t>(ws) & 3u))
+        return MOCE_ERR_INVALID_VALUE;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t *words = static_cast<uint32_t *>(ws);
+    cudaError_t err = launch_pack(C_in, C_out, k, support_idx, support_logits, packed_idx,
+                                  packed_logits, resid_idx, words, s);
+    if (err != cudaSuccess) return MOCE_ERR_CUDA;
+    uint32_t head[2] = {0u, 0u};
+    err = cudaMemcpyAsync(head, words, sizeof(head), cudaMemcpyDeviceToHost, s);
+    if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+    if (err != cudaSuccess) return MOCE_ERR_CUDA;
+    if (head[0] != 0u) return MOCE_ERR_BAD_SUPPORT;
+    *n_resid_host = (int32_t)head[1];
+    return MOCE_OK;
+}
+
+size_t moce_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k) {
+    if (!shape_ok(N, H, W, C_in, C_out, k)) return 0;
+    return ws_layout(N, H * W, C_in, C_out, k).total;
+}
+
+moce_status_t moce_workspace_init(void *ws, size_t ws_bytes, moce_stream_t stream) {
+    if (!ws) return MOCE_ERR_INVALID_VALUE;
+    return cuda_status(cudaMemsetAsync(ws, 0, ws_bytes, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+moce_status_t moce_workspace_offsets(int N, int H, int W, int C_in, int C_out, int k,
+                                     size_t *z_offset, size_t *tau_offset) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !z_offset || !tau_offset)
+        return MOCE_ERR_INVALID_VALUE;
+    const WsLayout L = ws_layout(N, H * W, C_in, C_out, k);
+    *z_offset = L.z;
+    *tau_offset = L.tau;
+    return MOCE_OK;
+}
+
+moce_status_t moce_pool(const void *x, int N, int H, int W, int C_in, moce_dtype_t dtype,
+                        moce_layout_t layout, float *z, void *ws, size_t ws_bytes,
+                        moce_stream_t stream) {
+    if (!shape_ok(N, H, W, C_in, 1, 1) || !dtype_ok(dtype) || !layout_ok(layout))
+        return MOCE_ERR_INVALID_VALUE;
+    if (N > 0 && (H * W < 1 || !x || !z || !ws)) return MOCE_ERR_INVALID_VALUE;
+    const WsLayout L = ws_layout(N, H * W, C_in, 1, 1);
+    if (layout == MOCE_NHWC && ws_bytes < L.total) return MOCE_ERR_INVALID_VALUE;
+    if (reinterpret_cast<uintptr_t>(ws) & 255u) return MOCE_ERR_INVALID_VALUE;
+    return cuda_status(launch_pool(x, N, H * W, C_in, dtype, layout, z, L,
+                                   static_cast<unsigned char *>(ws),
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
+                        const int32_t *packed_idx, const float *packed_logits, const float *W1,
+                        const float *b1, const float *w2, const float *b2, float tau_min,
+                        float tau_max, float *tau, float *mix_w, moce_stream_t stream) {
+    if (!shape_ok(N, 1, 1, C_in, C_out, k) || !tau_ok(tau_min, tau_max))
+        return MOCE_ERR_INVALID_VALUE;
+    if (N > 0 && (!z || !packed_idx || !packed_logits || !W1 || !b1 || !w2 || !b2 || !tau))
+        return MOCE_ERR_INVALID_VALUE;
+    if (gate_smem_bytes(k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    return cuda_status(launch_gate(z, N, C_in, C_out, k, packed_idx, packed_logits, W1, b1, w2, b2,
+                                   tau_min, tau_max, tau, mix_w,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                           moce_dtype_t dtype, moce_layout_t layout, const int32_t *packed_idx,
+                           const float *packed_logits, const int32_t *resid_idx, int n_resid,
+                           const float *W1, const float *b1, const float *w2, const float *b2,
+                           float tau_min, float tau_max, void *y, void *ws, size_t ws_bytes,
+                           moce_stream_t stream) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
+        !tau_ok(tau_min, tau_max))
+        return MOCE_ERR_INVALID_VALUE;
+    if (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
+    const int HW = H * W;
+    if (N == 0 || HW == 0) return MOCE_OK;
+    if (!x || !packed_idx || !packed_logits || !W1 || !b1 || !w2 || !b2 || !y || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    const WsLayout L = ws_layout(N, HW, C_in, C_out, k);
+    if (ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MOCE_ERR_INVALID_VALUE;
+    if (gate_smem_bytes(k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    unsigned char *wsb = static_cast<unsigned char *>(ws);
+    float *z = reinterpret_cast<float *>(wsb + L.z);
+    float *tau = reinterpret_cast<float *>(wsb + L.tau);
+    float *a = reinterpret_cast<float *>(wsb + L.a);
+    if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
+        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_supported(N, HW, C_in, C_out, k)) {
+        return cuda_status(launch_fused(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
+                                        packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
+                                        b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
+                                        s));
+    }
+    cudaError_t err = launch_pool(x, N, HW, C_in, dtype, layout, z, L, wsb, s);
+    if (err == cudaSuccess)
+        err = launch_gate(z, N, C_in, C_out, k, packed_idx, packed_logits, W1, b1, w2, b2, tau_min,
+                          tau_max, tau, a, s);
+    if (err == cudaSuccess)
+        err = launch_mix(x, N, HW, C_in, C_out, k, dtype, layout, packed_idx, a, resid_idx,
+                         n_resid, y, s);
+    return cuda_status(err);
+}
+
+moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {
+    if (!ws || ws_bytes < kCtrlWords * 4) return MOCE_ERR_INVALID_VALUE;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t words[kCtrlWords];
+    cudaError_t err = cudaMemcpyAsync(words, ws, sizeof(words), cudaMemcpyDeviceToHost, s);
+    if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+    if (err != cudaSuccess) return MOCE_ERR_CUDA;
+    return words[kCtrlError] ? MOCE_ERR_TIMEOUT : MOCE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,128 @@
+// Internal declarations of the MoCE CUDA library (sm_103a). Not part of the ABI.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "moce.h"
+
+namespace moce {
+
+constexpr int kThreads = 256;
+
+__host__ __device__ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ---------------------------------------------------------------- workspace
+// Control words at the start of a forward workspace.
+enum CtrlWord : int {
+    kCtrlWorkCounter = 0,  // next work item of the fused persistent kernel
+    kCtrlExitCounter = 1,  // CTAs that finished the fused kernel
+    kCtrlEpoch = 2,        // number of completed fused forwards (flag values are epoch + 1)
+    kCtrlError = 3,        // 0, or kErrTimeout
+    kCtrlErrorItem = 4,    // work item whose wait gave up
+    kCtrlWords = 64
+};
+constexpr uint32_t kErrTimeout = 1u;
+
+// Pixels per pooling tile: about 64 KB of bf16 input per tile.
+inline int pool_tile_px(int C) {
+    int pp = 32768 / (C > 0 ? C : 1);
+    int p2 = 4;
+    while (p2 * 2 <= pp && p2 < 256) p2 *= 2;
+    return p2;
+}
+
+struct WsLayout {
+    size_t ctrl = 0;      // kCtrlWords uint32
+    size_t ticket = 0;    // [N] uint32: pooling tiles finished
+    size_t gcount = 0;    // [N] uint32: gate blocks finished
+    size_t zflag = 0;     // [N] uint32: epoch + 1 once z[n] is complete
+    size_t gflag = 0;     // [N] uint32: epoch + 1 once tau[n], a[n] are complete
+    size_t partial = 0;   // [N][pool_tiles][C] fp32 pooling partial sums
+    size_t z = 0;         // [N][C] fp32
+    size_t tau = 0;       // [N][R] fp32
+    size_t a = 0;         // [N][R][k] fp32 mixing weights
+    size_t total = 0;
+    int pool_px = 0;
+    int pool_tiles = 0;
+};
+
+inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
+    WsLayout L;
+    L.pool_px = pool_tile_px(C);
+    L.pool_tiles = (HW + L.pool_px - 1) / L.pool_px;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+    L.ctrl = take(kCtrlWords * 4);
+    L.ticket = take((size_t)N * 4);
+    L.gcount = take((size_t)N * 4);
+    L.zflag = take((size_t)N * 4);
+    L.gflag = take((size_t)N * 4);
+    L.partial = take((size_t)N * L.pool_tiles * C * 4);
+    L.z = take((size_t)N * C * 4);
+    L.tau = take((size_t)N * R * 4);
+    L.a = take((size_t)N * R * k * 4);
+    L.total = off;
+    return L;
+}
+
+// ---------------------------------------------------------------- device helpers
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+__device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
+__device__ __forceinline__ uint16_t f32_to_bf16(float f) {
+    return __bfloat16_as_ushort(__float2bfloat16_rn(f));
+}
+
+template <typename T> __device__ __forceinline__ float load_elem(const T *p);
+template <> __device__ __forceinline__ float load_elem<float>(const float *p) { return __ldg(p); }
+template <> __device__ __forceinline__ float load_elem<uint16_t>(const uint16_t *p) {
+    return bf16_to_f32(__ldg(p));
+}
+template <typename T> __device__ __forceinline__ T store_cvt(float v);
+template <> __device__ __forceinline__ float store_cvt<float>(float v) { return v; }
+template <> __device__ __forceinline__ uint16_t store_cvt<uint16_t>(float v) { return f32_to_bf16(v); }
+
+// ---------------------------------------------------------------- tiled mix geometry
+// The NHWC bf16 mixing kernels stage a tile of TP = 8*GS pixels of one
+// example in shared memory, transposed to channel-major rows of TP bf16
+// (pixel pairs packed in 32-bit words); groups of GS lanes each own 8 pixels
+// per lane and mix whole experts (or 1/S of an expert).
+struct MixGeom {
+    int GS = 0, TP = 0, G = 0;  // lanes per group, pixels per tile, groups per CTA
+    int EB = 0;                 // experts per table chunk
+    int S = 1;                  // parts each expert's k entries are split into
+    int kp = 0;                 // k rounded up to even (entries per expert in the table)
+    int kq = 0;                 // entries per part (even)
+    size_t off_ys = 0, off_rp = 0, off_pp = 0, off_tab = 0, smem = 0;
+};
+
+bool mix_geometry(int C, int R, int k, size_t smem_budget, MixGeom *g);
+
+// ---------------------------------------------------------------- launchers (host)
+cudaError_t launch_pack(int C, int R, int k, const int32_t *idx, const float *lg, int32_t *pidx,
+                        float *plog, int32_t *resid, uint32_t *ws_words, cudaStream_t s);
+
+cudaError_t launch_pool(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay,
+                        float *z, const WsLayout &L, unsigned char *ws, cudaStream_t s);
+
+cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_t *pidx,
+                        const float *plog, const float *W1, const float *b1, const float *w2,
+                        const float *b2, float tmin, float tmax, float *tau, float *a,
+                        cudaStream_t s);
+
+cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
+                       moce_layout_t lay, const int32_t *pidx, const float *a,
+                       const int32_t *resid, int nU, void *y, cudaStream_t s);
+
+cudaError_t launch_fused(const uint16_t *x, int N, int HW, int C, int R, int k,
+                         const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
+                         const float *W1, const float *b1, const float *w2, const float *b2,
+                         float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
+                         cudaStream_t s);
+
+bool fused_supported(int N, int HW, int C, int R, int k);
+
+}  // namespace moce

@@ -1,0 +1,230 @@
+"""Python binding of the MoCE C ABI (include/moce.h).
+
+Argument marshalling only: every step of the layer runs in the CUDA kernels
+of ``libmoce.so``. PyTorch provides device memory and the current stream.
+There is no CPU fallback: if the library is not built, or a tensor is not on
+a CUDA device, the call raises.
+
+The functions carry the C names. Tensors:
+  x              NHWC [N, H, W, C_in] or NCHW [N, C_in, H, W]; torch.bfloat16 or float32
+  y              same layout/dtype with C_out + 1 channels (residual expert last)
+  support_idx    int32 [C_out, k]; support_logits float32 [C_out, k]
+  W1 [k, k] (row j = hidden unit j), b1 [k], w2 [k], b2 [1]: float32
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+from . import build as _build
+
+MOCE_OK, MOCE_ERR_INVALID_VALUE, MOCE_ERR_BAD_SUPPORT = 0, 1, 2
+MOCE_ERR_UNSUPPORTED, MOCE_ERR_CUDA, MOCE_ERR_TIMEOUT = 3, 4, 5
+MOCE_F32, MOCE_BF16 = 0, 1
+MOCE_NHWC, MOCE_NCHW = 0, 1
+_LAYOUTS = {"nhwc": MOCE_NHWC, "nchw": MOCE_NCHW}
+
+_lib = None
+
+
+class MoceError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        name = library().moce_status_string(status).decode()
+        super().__init__(f"{what} failed: {name}")
+        self.status = status
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def library():
+    """The loaded ``libmoce.so`` (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        path = library_path()
+        if not os.path.exists(path):
+            raise RuntimeError(f"MoCE CUDA library not built ({path}); run "
+                               "paper_2608_23794_gb300.build.build() first")
+        lib = ctypes.CDLL(path)
+        P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+        sig = {
+            "moce_status_string": ([I], ctypes.c_char_p),
+            "moce_pack_workspace_bytes": ([I, I, I], S),
+            "moce_pack_supports": ([I, I, I, P, P, P, P, P, P, P, S, P], I),
+            "moce_workspace_bytes": ([I, I, I, I, I, I], S),
+            "moce_workspace_init": ([P, S, P], I),
+            "moce_workspace_offsets": ([I, I, I, I, I, I, P, P], I),
+            "moce_pool": ([P, I, I, I, I, I, I, P, P, S, P], I),
+            "moce_gate": ([P, I, I, I, I, P, P, P, P, P, P, F, F, P, P, P], I),
+            "moce_forward": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S, P], I),
+            "moce_check_device_error": ([P, S, P], I),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes, fn.restype = args, res
+        _lib = lib
+    return _lib
+
+
+def _check(status: int, what: str):
+    if status != MOCE_OK:
+        raise MoceError(status, what)
+
+
+def _ptr(t: torch.Tensor | None):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("MoCE tensors must be CUDA tensors")
+    if not t.is_contiguous():
+        raise ValueError("MoCE tensors must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream: torch.cuda.Stream | None = None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return MOCE_BF16
+    if t.dtype == torch.float32:
+        return MOCE_F32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _dims(x: torch.Tensor, layout: str):
+    if layout == "nhwc":
+        N, H, W, C = x.shape
+    elif layout == "nchw":
+        N, C, H, W = x.shape
+    else:
+        raise ValueError(layout)
+    return N, H, W, C
+
+
+@dataclass
+class PackedSupports:
+    packed_idx: torch.Tensor      # int32 [C_out, k], rows in deployment order
+    packed_logits: torch.Tensor   # float32 [C_out, k]
+    resid_idx: torch.Tensor       # int32 [C_in]; the first n_resid entries are U
+    n_resid: int
+    C_in: int
+
+    @property
+    def C_out(self) -> int:
+        return self.packed_idx.shape[0]
+
+    @property
+    def k(self) -> int:
+        return self.packed_idx.shape[1]
+
+
+def moce_pack_supports(support_idx: torch.Tensor, support_logits: torch.Tensor, C_in: int,
+                       stream=None) -> PackedSupports:
+    R, k = support_idx.shape
+    dev = support_idx.device
+    out_idx = torch.empty((R, k), dtype=torch.int32, device=dev)
+    out_lg = torch.empty((R, k), dtype=torch.float32, device=dev)
+    resid = torch.empty((C_in,), dtype=torch.int32, device=dev)
+    ws_bytes = library().moce_pack_workspace_bytes(C_in, R, k)
+    if ws_bytes == 0:
+        raise MoceError(MOCE_ERR_INVALID_VALUE, "moce_pack_workspace_bytes")
+    ws = torch.empty((ws_bytes,), dtype=torch.uint8, device=dev)
+    n_resid = ctypes.c_int32(0)
+    _check(library().moce_pack_supports(C_in, R, k, _ptr(support_idx.to(torch.int32).contiguous()),
+                                        _ptr(support_logits.to(torch.float32).contiguous()),
+                                        _ptr(out_idx), _ptr(out_lg), _ptr(resid),
+                                        ctypes.byref(n_resid), _ptr(ws), ws_bytes, _stream(stream)),
+           "moce_pack_supports")
+    return PackedSupports(out_idx, out_lg, resid, int(n_resid.value), C_in)
+
+
+def moce_workspace_bytes(N: int, H: int, W: int, C_in: int, C_out: int, k: int) -> int:
+    return int(library().moce_workspace_bytes(N, H, W, C_in, C_out, k))
+
+
+class Workspace:
+    """A zero-initialised forward workspace for one layer shape."""
+
+    def __init__(self, N, H, W, C_in, C_out, k, device="cuda"):
+        self.shape = (N, H, W, C_in, C_out, k)
+        nbytes = moce_workspace_bytes(N, H, W, C_in, C_out, k)
+        if nbytes == 0:
+            raise MoceError(MOCE_ERR_INVALID_VALUE, "moce_workspace_bytes")
+        self.buffer = torch.zeros((nbytes,), dtype=torch.uint8, device=device)
+        z_off, tau_off = ctypes.c_size_t(0), ctypes.c_size_t(0)
+        _check(library().moce_workspace_offsets(N, H, W, C_in, C_out, k, ctypes.byref(z_off),
+                                                ctypes.byref(tau_off)), "moce_workspace_offsets")
+        self.z_offset, self.tau_offset = z_off.value, tau_off.value
+
+    @property
+    def nbytes(self) -> int:
+        return self.buffer.numel()
+
+    def z(self) -> torch.Tensor:
+        N, _, _, C, _, _ = self.shape
+        return self.buffer[self.z_offset:self.z_offset + 4 * N * C].view(torch.float32).view(N, C)
+
+    def tau(self) -> torch.Tensor:
+        N, _, _, _, R, _ = self.shape
+        return self.buffer[self.tau_offset:self.tau_offset + 4 * N * R].view(torch.float32).view(N, R)
+
+    def init(self, stream=None):
+        _check(library().moce_workspace_init(_ptr(self.buffer), self.nbytes, _stream(stream)),
+               "moce_workspace_init")
+
+
+def moce_pool(x: torch.Tensor, layout: str, ws: Workspace | None = None, z=None,
+              stream=None) -> torch.Tensor:
+    N, H, W, C = _dims(x, layout)
+    if z is None:
+        z = torch.empty((N, C), dtype=torch.float32, device=x.device)
+    if ws is None:
+        ws = Workspace(N, H, W, C, 1, 1, device=x.device)
+    _check(library().moce_pool(_ptr(x), N, H, W, C, _dtype(x), _LAYOUTS[layout], _ptr(z),
+                               _ptr(ws.buffer), ws.nbytes, _stream(stream)), "moce_pool")
+    return z
+
+
+def moce_gate(z: torch.Tensor, packed: PackedSupports, W1, b1, w2, b2, tau_min: float,
+              tau_max: float, want_weights: bool = True, stream=None):
+    N, C = z.shape
+    R, k = packed.C_out, packed.k
+    tau = torch.empty((N, R), dtype=torch.float32, device=z.device)
+    a = torch.empty((N, R, k), dtype=torch.float32, device=z.device) if want_weights else None
+    _check(library().moce_gate(_ptr(z), N, C, R, k, _ptr(packed.packed_idx),
+                               _ptr(packed.packed_logits), _ptr(W1), _ptr(b1), _ptr(w2), _ptr(b2),
+                               float(tau_min), float(tau_max), _ptr(tau), _ptr(a),
+                               _stream(stream)), "moce_gate")
+    return tau, a
+
+
+def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
+                 tau_min: float, tau_max: float, ws: Workspace | None = None,
+                 y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    N, H, W, C = _dims(x, layout)
+    R, k = packed.C_out, packed.k
+    if C != packed.C_in:
+        raise ValueError("x channels do not match the packed supports")
+    if y is None:
+        shape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+        y = torch.empty(shape, dtype=x.dtype, device=x.device)
+    if ws is None:
+        ws = Workspace(N, H, W, C, R, k, device=x.device)
+    _check(library().moce_forward(_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout],
+                                  _ptr(packed.packed_idx), _ptr(packed.packed_logits),
+                                  _ptr(packed.resid_idx), packed.n_resid, _ptr(W1), _ptr(b1),
+                                  _ptr(w2), _ptr(b2), float(tau_min), float(tau_max), _ptr(y),
+                                  _ptr(ws.buffer), ws.nbytes, _stream(stream)), "moce_forward")
+    return y
+
+
+def moce_check_device_error(ws: Workspace, stream=None):
+    _check(library().moce_check_device_error(_ptr(ws.buffer), ws.nbytes, _stream(stream)),
+           "moce_check_device_error")

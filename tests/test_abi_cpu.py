@@ -1,0 +1,107 @@
+"""The C ABI library builds, loads and exports every declared entry point;
+host-side validation rejects bad arguments before touching any GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_23794_gb300 import build as moce_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moce.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = moce_build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(moce_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("moce_pack_supports", "moce_pool", "moce_gate", "moce_forward",
+                     "moce_workspace_bytes", "moce_status_string", "moce_check_device_error"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    lib.moce_status_string.restype = ctypes.c_char_p
+    lib.moce_status_string.argtypes = [ctypes.c_int]
+    assert lib.moce_status_string(0) == b"MOCE_OK"
+    assert lib.moce_status_string(2) == b"MOCE_ERR_BAD_SUPPORT"
+    assert lib.moce_status_string(99) == b"MOCE_ERR_UNKNOWN"
+
+
+def test_workspace_bytes(lib):
+    f = lib.moce_workspace_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_int] * 6
+    n = f(64, 56, 56, 256, 64, 16)
+    # z + tau + mixing weights + pooling partials at least
+    assert n >= 64 * 256 * 4 + 64 * 64 * 4 + 64 * 64 * 16 * 4
+    assert n % 256 == 0
+    assert f(64, 56, 56, 256, 64, 0) == 0          # k < 1
+    assert f(64, 56, 56, 256, 64, 257) == 0        # k > C_in
+    assert f(1, 1, 1, 70000, 4, 2) == 0            # C_in beyond 16-bit indices
+    pf = lib.moce_pack_workspace_bytes
+    pf.restype = ctypes.c_size_t
+    pf.argtypes = [ctypes.c_int] * 3
+    assert pf(256, 64, 16) >= 4 * (2 + 256 // 32)
+
+
+def test_forward_rejects_bad_arguments_on_host(lib):
+    f = lib.moce_forward
+    P, I, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    f.argtypes = [P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, ctypes.c_size_t, P]
+    f.restype = I
+    fake = ctypes.c_void_p(0x1000)  # never dereferenced: validation fails first
+    good = dict(x=fake, N=2, H=4, W=4, C=64, R=8, k=4, dt=1, lay=0, tmin=0.2, tmax=6.0)
+
+    def call(**kw):
+        a = {**good, **kw}
+        return f(a["x"], a["N"], a["H"], a["W"], a["C"], a["R"], a["k"], a["dt"], a["lay"], fake,
+                 fake, fake, 3, fake, fake, fake, fake, a["tmin"], a["tmax"], fake, fake, 0, None)
+
+    assert call(k=0) == 1
+    assert call(k=65) == 1
+    assert call(R=0) == 1
+    assert call(dt=7) == 1
+    assert call(lay=3) == 1
+    assert call(tmin=0.0) == 1
+    assert call(tmin=7.0) == 1
+    assert call(tmax=float("inf")) == 1
+    assert call(x=None) == 1
+    assert call() == 1  # workspace of 0 bytes is too small
+    assert call(N=0) == 0  # empty batch: nothing to do
+
+
+def test_pack_rejects_bad_arguments_on_host(lib):
+    f = lib.moce_pack_supports
+    P, I = ctypes.c_void_p, ctypes.c_int
+    f.argtypes = [I, I, I, P, P, P, P, P, P, P, ctypes.c_size_t, P]
+    f.restype = I
+    fake = ctypes.c_void_p(0x1000)
+    n = ctypes.c_int32(0)
+    assert f(64, 8, 0, fake, fake, fake, fake, fake, ctypes.byref(n), fake, 4096, None) == 1
+    assert f(64, 8, 4, None, fake, fake, fake, fake, ctypes.byref(n), fake, 4096, None) == 1
+    assert f(64, 8, 4, fake, fake, fake, fake, fake, ctypes.byref(n), fake, 4, None) == 1
+
+
+def test_binding_refuses_cpu_tensors():
+    torch = pytest.importorskip("torch")
+    from paper_2608_23794_gb300 import moce
+    x = torch.zeros((1, 2, 2, 8), dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        moce._ptr(x)
