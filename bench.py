@@ -1,0 +1,432 @@
+#!/usr/bin/env python
+"""MoCE layer forward benchmark on GB300.
+
+One step = one MoCE forward (pooling, gate, softmax weights, routed mixing,
+residual) over the whole batch of the ResNet-50 stage-1 bottleneck-entrance
+projection (N=64, 56x56, C_in=256 -> 64 routed experts + 1 residual, k=16,
+bf16 NHWC), on seeded synthetic inputs already resident in HBM. Supports are
+packed once before timing (reported separately as pack_us).
+
+Reported value: achieved algorithmic HBM bandwidth, GB/s = (x read once +
+y written once + packed tables + gate parameters) / layer time, summed over
+ranks and divided by the slowest rank's time. us_per_layer is the layer time.
+Between timed steps the inputs rotate over enough copies that every step
+reads x from HBM, not L2.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (the plain restatement of the paper's
+equations) on the host cores, on a bounded sample of the same workload.
+Multi-GPU (torchrun): every rank runs its own batch (weak scaling, no
+collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "rn50_stage1_reduce"
+METRIC = "MoCE fwd µs/layer & achieved HBM GB/s (% of GB300 peak) vs dense 1×1 cuBLAS"
+UNIT = "GB/s"
+SEED = 0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="CPU work budget of the oracle baseline leg")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ helpers
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def workload_bytes(cfg, n_resid: int) -> int:
+    from paper_2608_23794_gb300 import costmodel
+    return costmodel.layer_bytes(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k,
+                                 cfg.elem_bytes, n_resid)
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def csrc_hash() -> str:
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2608_23794_gb300", "csrc")
+    for f in sorted(os.listdir(d)):
+        with open(os.path.join(d, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if taken on the current kernels."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    rec = d.get(workload)
+    if not rec or rec.get("csrc_hash") != csrc_hash():
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples taken while the timed region runs."""
+
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.lines: list[str] = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        rows = []
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 10:
+                continue
+            if self.uuid and parts[1] != self.uuid:
+                continue
+            rows.append(parts)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[6 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def gpu_uuid(torch, dev):
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------------ CPU oracle leg
+
+
+def oracle_sample_run(lay, cfg, budget_s: float):
+    """Time the oracle on a bounded sample of the workload; returns (GB/s, sample str, reps)."""
+    import numpy as np
+
+    import oracle
+    pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, cfg.C_in)
+    args = (pidx, plog, resid, lay.W1, lay.b1, lay.w2, float(lay.b2[0]), cfg.tau_min, cfg.tau_max)
+    # one example first, to size the sample
+    t0 = time.perf_counter()
+    oracle.forward(lay.x[:1], cfg.layout, *args)
+    t_ex = max(time.perf_counter() - t0, 1e-6)
+    n_ex = int(max(1, min(cfg.N, budget_s / t_ex)))
+    h_rows = cfg.H
+    if t_ex > budget_s and cfg.layout == "nhwc":
+        h_rows = int(max(1, cfg.H * budget_s / t_ex))
+    xs = np.ascontiguousarray(lay.x[:n_ex, :h_rows]) if cfg.layout == "nhwc" else lay.x[:n_ex]
+    reps, times = 0, []
+    start = time.perf_counter()
+    while True:
+        t0 = time.perf_counter()
+        oracle.forward(xs, cfg.layout, *args)
+        times.append(time.perf_counter() - t0)
+        reps += 1
+        if time.perf_counter() - start >= budget_s or reps >= 1000:
+            break
+    sub = cfg.replace(N=n_ex, H=h_rows)
+    nbytes = workload_bytes(sub, len(resid))
+    t = statistics.median(times)
+    sample = (f"{n_ex} of {cfg.N} examples x {h_rows} of {cfg.H} rows, median of {reps} "
+              f"single-threaded oracle runs")
+    return nbytes / t / 1e9, sample, t
+
+
+def run_reference(args, cfg):
+    """The reference arm: the CPU oracle, timed as it stands, on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2608_23794_gb300 import synth
+    import oracle
+    oracle.build()
+    lay = synth.make_layer(cfg, seed=SEED)
+    pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, cfg.C_in)
+    args_o = (pidx, plog, resid, lay.W1, lay.b1, lay.w2, float(lay.b2[0]), cfg.tau_min, cfg.tau_max)
+    t0 = time.perf_counter()
+    oracle.forward(lay.x[:1], cfg.layout, *args_o)
+    t_ex = max(time.perf_counter() - t0, 1e-6)
+    # each step is a bounded sample so that warmup + steps fit in about two minutes
+    per_step = 120.0 / max(1, args.steps + args.warmup)
+    n_ex = int(max(1, min(cfg.N, per_step / t_ex)))
+    h_rows = cfg.H if t_ex <= per_step else int(max(1, cfg.H * per_step / t_ex))
+    xs = lay.x[:n_ex, :h_rows].copy()
+    for _ in range(args.warmup):
+        oracle.forward(xs, cfg.layout, *args_o)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.forward(xs, cfg.layout, *args_o)
+    dt = (time.perf_counter() - t0) / max(1, args.steps)
+    sub = cfg.replace(N=n_ex, H=h_rows)
+    value = workload_bytes(sub, len(resid)) / dt / 1e9
+    sample = f"{n_ex} of {cfg.N} examples x {h_rows} of {cfg.H} rows per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; stands in for ImageNet activations)",
+        "config": {"workload": cfg.name, "N": cfg.N, "H": cfg.H, "W": cfg.W, "C_in": cfg.C_in,
+                   "C_out": cfg.C_out, "k": cfg.k, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ our arm
+
+
+def run_ours(args, cfg):
+    import numpy as np
+    import torch
+
+    from paper_2608_23794_gb300 import build as moce_build
+    from paper_2608_23794_gb300 import costmodel, moce, synth
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    moce_build.build()
+
+    lay = synth.make_layer(cfg, seed=SEED + rank)
+    bits = torch.from_numpy(lay.x_bits.view(np.int16)).view(torch.bfloat16)
+    cu = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).to(device=dev, dtype=dt)
+    W1, b1, w2, b2 = (cu(lay.W1, torch.float32), cu(lay.b1, torch.float32),
+                      cu(lay.w2, torch.float32), cu(lay.b2, torch.float32))
+    sidx, slog = cu(lay.support_idx, torch.int32), cu(lay.support_logits, torch.float32)
+
+    # one-time packing (Sec. 3.2: supports are static at inference)
+    moce.moce_pack_supports(sidx, slog, cfg.C_in)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    packed = moce.moce_pack_supports(sidx, slog, cfg.C_in)
+    e1.record()
+    torch.cuda.synchronize()
+    pack_us = e0.elapsed_time(e1) * 1e3
+
+    # rotate input/output copies so that every timed step reads x from HBM
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 132 * 2**20
+    x_bytes = bits.numel() * 2
+    n_rot = max(2, int(np.ceil(3 * l2 / x_bytes)) + 1)
+    xs = [bits.to(dev) for _ in range(n_rot)]
+    ys = [torch.empty((cfg.N, cfg.H, cfg.W, cfg.C_out + 1), dtype=torch.bfloat16, device=dev)
+          for _ in range(n_rot)]
+    ws = moce.Workspace(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k, device=dev)
+    fwd = lambda i: moce.moce_forward(xs[i % n_rot], "nhwc", packed, W1, b1, w2, b2, cfg.tau_min,
+                                      cfg.tau_max, ws=ws, y=ys[i % n_rot])
+    launches_per_step = moce.moce_forward_launches(xs[0], "nhwc", cfg.C_out, cfg.k)
+
+    for i in range(args.warmup):
+        fwd(i)
+    torch.cuda.synchronize()
+    moce.moce_check_device_error(ws)
+
+    K = args.steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(gpu_uuid(torch, dev))
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_begin.record()
+    for i in range(K):
+        starts[i].record()
+        fwd(i)
+        ends[i].record()
+    t_end.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop()
+    moce.moce_check_device_error(ws)
+    total_ms = t_begin.elapsed_time(t_end)
+    launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / K
+    nbytes = workload_bytes(cfg, packed.n_resid)
+    value = nbytes * world * K / (total_ms * 1e-3) / 1e9
+
+    # roofline of the dominant kernel (the whole forward when it is one fused launch)
+    peaks, peak_src = measured_peaks()
+    kern_s = statistics.mean(launch_ms) * 1e-3
+    achieved = nbytes / kern_s / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "traffic": ncu_traffic(cfg.name),
+                "peak_source": f"{peak_src} (burst copy)", "kernel": (
+                    "moce_fused_forward" if launches_per_step == 1 else
+                    f"moce_forward ({launches_per_step} launches)"),
+                "algorithmic_bytes_per_launch": nbytes}
+
+    # dense 1x1 comparator: cuBLAS bf16 GEMM [P x C_in] x [C_in x C_out]
+    P = cfg.N * cfg.H * cfg.W
+    Wd = torch.randn(cfg.C_in, cfg.C_out, device=dev, dtype=torch.bfloat16)
+    outs = [torch.empty(P, cfg.C_out, device=dev, dtype=torch.bfloat16) for _ in range(n_rot)]
+    for i in range(20):
+        torch.matmul(xs[i % n_rot].view(P, cfg.C_in), Wd, out=outs[i % n_rot])
+    torch.cuda.synchronize()
+    Kd = min(K, 2000)
+    e0.record()
+    for i in range(Kd):
+        torch.matmul(xs[i % n_rot].view(P, cfg.C_in), Wd, out=outs[i % n_rot])
+    e1.record()
+    torch.cuda.synchronize()
+    dense_us = e0.elapsed_time(e1) * 1e3 / Kd
+    dense_bytes = P * cfg.C_in * 2 + P * cfg.C_out * 2 + cfg.C_in * cfg.C_out * 2
+
+    # end to end through the public API: pinned host x -> device, forward, y -> pinned host
+    x_host = bits.pin_memory()
+    y_host = torch.empty(ys[0].shape, dtype=torch.bfloat16).pin_memory()
+    x_dev, y_dev = xs[0], ys[0]
+    Ke = max(3, min(K, 200))
+    for _ in range(3):
+        x_dev.copy_(x_host, non_blocking=True)
+        moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
+                          y=y_dev)
+        y_host.copy_(y_dev, non_blocking=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(Ke):
+        x_dev.copy_(x_host, non_blocking=True)
+        moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
+                          y=y_dev)
+        y_host.copy_(y_dev, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_s = e0.elapsed_time(e1) * 1e-3 / Ke
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = {"value": nbytes * world / e2e_s / 1e9, "unit": UNIT,
+           "h2d_bytes_per_step": x_bytes, "d2h_bytes_per_step": y_host.numel() * 2,
+           "us_per_layer": e2e_s * 1e6}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        gbs, sample, t_rep = oracle_sample_run(lay, cfg, args.cpu_seconds)
+        cpu = {"value": gbs, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        flops = costmodel.layer_flops(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k,
+                                      packed.n_resid)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "us_per_layer": ms_per_step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic (seeded post-ReLU N(0,1); stands in for ImageNet "
+                                    "activations)",
+            "config": {"workload": cfg.name, "N": cfg.N, "H": cfg.H, "W": cfg.W,
+                       "C_in": cfg.C_in, "C_out": cfg.C_out, "k": cfg.k, "n_resid": packed.n_resid,
+                       "storage_dtype": "bf16", "layout": "nhwc",
+                       "l2": f"inputs rotate over {n_rot} copies ({n_rot * x_bytes / 2**20:.0f} MiB"
+                             f" > 3x the {l2 / 2**20:.0f} MiB L2)",
+                       "parallelism": f"batch shard x{world} (no collective)"},
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step * K,
+            "clocks": clocks,
+            "pack_us": pack_us,
+            "dense_cublas": {"us_per_layer": dense_us, "GB/s": dense_bytes / dense_us / 1e3,
+                             "moce_speedup": dense_us / (ms_per_step * 1e3)},
+            "macs": {"routed": flops["routed_macs"], "gate": flops["gate_macs"],
+                     "dense_equiv": flops["dense_equiv_flops"] // 2},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    from paper_2608_23794_gb300 import synth
+    cfg = synth.CONFIGS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, cfg)
+    else:
+        run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    main()

@@ -170,6 +170,14 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
                            moce_stream_t stream);
 
 /*
+ * Number of kernel launches moce_forward makes for these arguments (the
+ * path selection depends on dtype, layout, C_in and the alignment of x).
+ * Returns 0 for arguments moce_forward would reject. Enqueues nothing.
+ */
+int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                          moce_dtype_t dtype, moce_layout_t layout);
+
+/*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word the
  * forward kernels leave in `ws` (a forward workspace). Returns MOCE_OK,
  * MOCE_ERR_TIMEOUT (a bounded inter-CTA wait gave up; outputs of that call

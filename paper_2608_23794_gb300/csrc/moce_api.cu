@@ -168,6 +168,17 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
     return cuda_status(err);
 }
 
+int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                          moce_dtype_t dtype, moce_layout_t layout) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout)) return 0;
+    if (N == 0 || H * W == 0) return 0;
+    if (gate_smem_bytes(k) > 227 * 1024) return 0;
+    if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
+        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_supported(N, H * W, C_in, C_out, k))
+        return 1;
+    return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
+}
+
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {
     if (!ws || ws_bytes < kCtrlWords * 4) return MOCE_ERR_INVALID_VALUE;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

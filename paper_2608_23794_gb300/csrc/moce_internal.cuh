@@ -10,21 +10,24 @@
 
 namespace moce {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 256;  // threads of the standalone kernels and of the fused kernel's mix group
 
 __host__ __device__ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 // ---------------------------------------------------------------- workspace
 // Control words at the start of a forward workspace.
 enum CtrlWord : int {
-    kCtrlWorkCounter = 0,  // next work item of the fused persistent kernel
-    kCtrlExitCounter = 1,  // CTAs that finished the fused kernel
-    kCtrlEpoch = 2,        // number of completed fused forwards (flag values are epoch + 1)
-    kCtrlError = 3,        // 0, or kErrTimeout
-    kCtrlErrorItem = 4,    // work item whose wait gave up
+    kCtrlExitCounter = 0,  // CTAs that finished the fused kernel
+    kCtrlEpoch = 1,        // number of completed fused forwards (data tags are epoch + 1)
+    kCtrlError = 2,        // 0, or kErrTimeout
+    kCtrlErrorItem = 3,    // 1 + the work item whose wait gave up
+    kCtrlDropItem = 4,     // fault injection for tests: 1 + a work item that must not publish
     kCtrlWords = 64
 };
 constexpr uint32_t kErrTimeout = 1u;
+
+// Experts per gate work item of the fused kernel.
+constexpr int kGateExperts = 64;
 
 // Pixels per pooling tile: about 64 KB of bf16 input per tile.
 inline int pool_tile_px(int C) {
@@ -36,34 +39,29 @@ inline int pool_tile_px(int C) {
 
 struct WsLayout {
     size_t ctrl = 0;      // kCtrlWords uint32
-    size_t ticket = 0;    // [N] uint32: pooling tiles finished
-    size_t gcount = 0;    // [N] uint32: gate blocks finished
-    size_t zflag = 0;     // [N] uint32: epoch + 1 once z[n] is complete
-    size_t gflag = 0;     // [N] uint32: epoch + 1 once tau[n], a[n] are complete
-    size_t partial = 0;   // [N][pool_tiles][C] fp32 pooling partial sums
+    size_t partial = 0;   // [N][pool_tiles][C] pooling tile sums: fp32 (multi-kernel path) or
+                          // tagged 64-bit words {fp32 bits, epoch + 1} (fused kernel)
     size_t z = 0;         // [N][C] fp32
     size_t tau = 0;       // [N][R] fp32
-    size_t a = 0;         // [N][R][k] fp32 mixing weights
+    size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit
     size_t total = 0;
     int pool_px = 0;
     int pool_tiles = 0;
+    int gate_blocks = 0;
 };
 
 inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     WsLayout L;
     L.pool_px = pool_tile_px(C);
     L.pool_tiles = (HW + L.pool_px - 1) / L.pool_px;
+    L.gate_blocks = (R + kGateExperts - 1) / kGateExperts;
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     L.ctrl = take(kCtrlWords * 4);
-    L.ticket = take((size_t)N * 4);
-    L.gcount = take((size_t)N * 4);
-    L.zflag = take((size_t)N * 4);
-    L.gflag = take((size_t)N * 4);
-    L.partial = take((size_t)N * L.pool_tiles * C * 4);
+    L.partial = take((size_t)N * L.pool_tiles * C * 8);
     L.z = take((size_t)N * C * 4);
     L.tau = take((size_t)N * R * 4);
-    L.a = take((size_t)N * R * k * 4);
+    L.a = take((size_t)N * R * k * 8);
     L.total = off;
     return L;
 }

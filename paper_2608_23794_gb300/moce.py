@@ -62,6 +62,7 @@ def library():
             "moce_gate": ([P, I, I, I, I, P, P, P, P, P, P, F, F, P, P, P], I),
             "moce_forward": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S, P], I),
             "moce_check_device_error": ([P, S, P], I),
+            "moce_forward_launches": ([P, I, I, I, I, I, I, I, I], I),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -223,6 +224,13 @@ def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w
                                   _ptr(w2), _ptr(b2), float(tau_min), float(tau_max), _ptr(y),
                                   _ptr(ws.buffer), ws.nbytes, _stream(stream)), "moce_forward")
     return y
+
+
+def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int) -> int:
+    """Kernel launches one moce_forward call makes for this input."""
+    N, H, W, C = _dims(x, layout)
+    return int(library().moce_forward_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
+                                                _LAYOUTS[layout]))
 
 
 def moce_check_device_error(ws: Workspace, stream=None):

@@ -98,12 +98,28 @@ class SyntheticLayer:
 
 def bf16_bits(a: np.ndarray) -> np.ndarray:
     """float32 -> bf16 bit patterns, round to nearest even (finite inputs)."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
-    return ((u + (((u >> 16) & 1) + 0x7FFF)) >> 16).astype(np.uint16)
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).reshape(-1)
+    out = np.empty(u.size, np.uint16)
+    step = 1 << 22
+    for s0 in range(0, u.size, step):
+        v = u[s0:s0 + step]
+        r = (v >> 16) & 1
+        r += 0x7FFF
+        r += v
+        r >>= 16
+        out[s0:s0 + step] = r
+    return out.reshape(np.shape(a))
 
 
 def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
-    return (bits.astype(np.uint32) << 16).view(np.float32)
+    b = np.ascontiguousarray(bits).reshape(-1)
+    out = np.empty(b.size, np.uint32)
+    step = 1 << 22
+    for s0 in range(0, b.size, step):
+        o = out[s0:s0 + step]
+        o[:] = b[s0:s0 + step]
+        o <<= 16
+    return out.view(np.float32).reshape(np.shape(bits))
 
 
 def _gelu(a: np.ndarray) -> np.ndarray:
