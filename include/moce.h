@@ -170,6 +170,31 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
                            moce_stream_t stream);
 
 /*
+ * The layer forward for callers that cannot allocate device memory: code
+ * running inside an allocator or memory-pool callback, loops that forbid
+ * allocation after start-up, plugins whose host framework owns every device
+ * buffer. The paper has no counterpart; it is a deployment convenience.
+ *
+ * Same arguments and results as moce_forward, without the workspace: the
+ * scratch is a fixed 8 MiB array in this library's device image (every GPU
+ * that loads the library holds it until the process exits). A layer whose
+ * moce_workspace_bytes exceeds 8 MiB is rejected with MOCE_ERR_UNSUPPORTED
+ * before anything is enqueued. The call itself allocates nothing.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture.
+ *   - Every call shares the one array per device: each call clears the part
+ *     it uses on `stream`, then runs the forward. Calls whose work overlaps on
+ *     the GPU (other streams, other host threads) race on the array.
+ */
+moce_status_t moce_forward_noalloc(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                   moce_dtype_t dtype, moce_layout_t layout,
+                                   const int32_t *packed_idx, const float *packed_logits,
+                                   const int32_t *resid_idx, int n_resid, const float *W1,
+                                   const float *b1, const float *w2, const float *b2,
+                                   float tau_min, float tau_max, void *y, moce_stream_t stream);
+
+/*
  * Number of kernel launches moce_forward makes for these arguments (the
  * path selection depends on dtype, layout, C_in and the alignment of x).
  * Returns 0 for arguments moce_forward would reject. Enqueues nothing.

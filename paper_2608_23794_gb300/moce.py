@@ -63,6 +63,7 @@ def library():
             "moce_forward": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S, P], I),
             "moce_check_device_error": ([P, S, P], I),
             "moce_forward_launches": ([P, I, I, I, I, I, I, I, I], I),
+            "moce_forward_noalloc": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P], I),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -231,6 +232,30 @@ def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int) -> i
     N, H, W, C = _dims(x, layout)
     return int(library().moce_forward_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
                                                 _LAYOUTS[layout]))
+
+
+def moce_forward_noalloc(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
+                         tau_min: float, tau_max: float, y: torch.Tensor | None = None,
+                         stream=None) -> torch.Tensor:
+    """moce_forward without a workspace, for callers that cannot allocate device memory.
+
+    The scratch is a fixed array inside the library (8 MiB per device); layers
+    that need more are rejected. Calls that overlap on the GPU share it and race.
+    """
+    N, H, W, C = _dims(x, layout)
+    R, k = packed.C_out, packed.k
+    if C != packed.C_in:
+        raise ValueError("x channels do not match the packed supports")
+    if y is None:
+        shape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+        y = torch.empty(shape, dtype=x.dtype, device=x.device)
+    _check(library().moce_forward_noalloc(_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout],
+                                          _ptr(packed.packed_idx), _ptr(packed.packed_logits),
+                                          _ptr(packed.resid_idx), packed.n_resid, _ptr(W1),
+                                          _ptr(b1), _ptr(w2), _ptr(b2), float(tau_min),
+                                          float(tau_max), _ptr(y), _stream(stream)),
+           "moce_forward_noalloc")
+    return y
 
 
 def moce_check_device_error(ws: Workspace, stream=None):
