@@ -59,10 +59,9 @@ def parse_args():
 
 
 def dist_env():
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return rank, world, local
+    from paper_2608_23794_gb300 import dist as mdist
+    info = mdist.rank_info()
+    return info.rank, info.world, info.local_rank
 
 
 def workload_bytes(cfg, n_resid: int) -> int:
@@ -260,7 +259,8 @@ def run_ours(args, cfg):
         dist.init_process_group("nccl", device_id=dev)
     moce_build.build()
 
-    lay = synth.make_layer(cfg, seed=SEED + rank)
+    from paper_2608_23794_gb300 import dist as mdist
+    lay = synth.make_layer(cfg, seed=mdist.shard_seed(SEED, rank))
     bits = torch.from_numpy(lay.x_bits.view(np.int16)).view(torch.bfloat16)
     cu = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).to(device=dev, dtype=dt)
     W1, b1, w2, b2 = (cu(lay.W1, torch.float32), cu(lay.b1, torch.float32),
@@ -317,13 +317,10 @@ def run_ours(args, cfg):
     moce.moce_check_device_error(ws)
     total_ms = t_begin.elapsed_time(t_end)
     launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = mdist.max_over_ranks(total_ms, device=dev)
     ms_per_step = total_ms / K
     nbytes = workload_bytes(cfg, packed.n_resid)
-    value = nbytes * world * K / (total_ms * 1e-3) / 1e9
+    value = mdist.job_throughput(nbytes * K, world, total_ms * 1e-3) / 1e9
 
     # roofline of the dominant kernel (the whole forward when it is one fused launch)
     peaks, peak_src = measured_peaks()
@@ -372,11 +369,8 @@ def run_ours(args, cfg):
     e1.record()
     torch.cuda.synchronize()
     e2e_s = e0.elapsed_time(e1) * 1e-3 / Ke
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e = {"value": nbytes * world / e2e_s / 1e9, "unit": UNIT,
+    e2e_s = mdist.max_over_ranks(e2e_s, device=dev)
+    e2e = {"value": mdist.job_throughput(nbytes, world, e2e_s) / 1e9, "unit": UNIT,
            "h2d_bytes_per_step": x_bytes, "d2h_bytes_per_step": y_host.numel() * 2,
            "us_per_layer": e2e_s * 1e6}
 
