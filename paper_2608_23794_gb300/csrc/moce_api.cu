@@ -151,8 +151,15 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
     float *z = reinterpret_cast<float *>(wsb + L.z);
     float *tau = reinterpret_cast<float *>(wsb + L.tau);
     float *a = reinterpret_cast<float *>(wsb + L.a);
-    if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
-        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_supported(N, HW, C_in, C_out, k)) {
+    const bool vec = dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
+                     (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+    if (vec && pipe_supported(N, HW, C_in, C_out, k)) {
+        return cuda_status(launch_pipe(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
+                                       packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
+                                       b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
+                                       s));
+    }
+    if (vec && fused_supported(N, HW, C_in, C_out, k)) {
         return cuda_status(launch_fused(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
                                         packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
                                         b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
@@ -174,7 +181,8 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
     if (N == 0 || H * W == 0) return 0;
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
     if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
-        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_supported(N, H * W, C_in, C_out, k))
+        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
+        (pipe_supported(N, H * W, C_in, C_out, k) || fused_supported(N, H * W, C_in, C_out, k)))
         return 1;
     return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
 }

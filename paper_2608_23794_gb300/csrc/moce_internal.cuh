@@ -29,9 +29,9 @@ constexpr uint32_t kErrTimeout = 1u;
 // Experts per gate work item of the fused kernel.
 constexpr int kGateExperts = 64;
 
-// Pixels per pooling tile: about 64 KB of bf16 input per tile.
+// Pixels per pooling tile: about 32 KB of bf16 input per tile.
 inline int pool_tile_px(int C) {
-    int pp = 32768 / (C > 0 ? C : 1);
+    int pp = 16384 / (C > 0 ? C : 1);
     int p2 = 4;
     while (p2 * 2 <= pp && p2 < 256) p2 *= 2;
     return p2;
@@ -40,7 +40,7 @@ inline int pool_tile_px(int C) {
 struct WsLayout {
     size_t ctrl = 0;      // kCtrlWords uint32
     size_t partial = 0;   // [N][pool_tiles][C] pooling tile sums: fp32 (multi-kernel path) or
-                          // tagged 64-bit words {fp32 bits, epoch + 1} (fused kernel)
+                          // tagged 64-bit words {fp32 bits, epoch + 1} (persistent kernels)
     size_t z = 0;         // [N][C] fp32
     size_t tau = 0;       // [N][R] fp32
     size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit
@@ -122,5 +122,13 @@ cudaError_t launch_fused(const uint16_t *x, int N, int HW, int C, int R, int k,
                          cudaStream_t s);
 
 bool fused_supported(int N, int HW, int C, int R, int k);
+
+cudaError_t launch_pipe(const uint16_t *x, int N, int HW, int C, int R, int k,
+                        const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
+                        const float *W1, const float *b1, const float *w2, const float *b2,
+                        float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
+                        cudaStream_t s);
+
+bool pipe_supported(int N, int HW, int C, int R, int k);
 
 }  // namespace moce
