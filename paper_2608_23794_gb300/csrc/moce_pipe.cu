@@ -53,6 +53,8 @@ constexpr int kPoolWarps = kPoolT / 32;
 constexpr int kGroups = kMixT / kGS;  // mixing groups per CTA
 constexpr int kRPS = kTP + 8;         // row stride (floats) of the residual partial sums
 constexpr int kBarStage = 2, kBarPrologue = 3;
+constexpr int kBufs = 2;              // tile buffers (x, y, residual sums) between stage and mix
+constexpr int kWTabs = kBufs + 1;     // per-run weight tables: the mix role may read kBufs runs
 constexpr int kStageU = 4;            // staging units (2 x 16 bytes) per stage thread and tile
 constexpr int kRun = 7;               // mixing tiles per run (one gate per run)
 constexpr int kPoolWin = 6;           // rolling window of 16-byte loads per pool thread
@@ -84,7 +86,7 @@ struct PipeParams {
     int cpw, rpi;                 // pool: 8-channel blocks per warp, rows per load instruction
     int kp, Es, ks, Kg, gate_tabs;  // Kg: padded gate width of the group gate, 0: warp gate
     int bulk_y;                   // output tiles leave by one bulk copy (rows of E = R + 1)
-    uint32_t off_xs[2], off_ys[2], off_rp[2], off_wst[3], off_offs;
+    uint32_t off_xs[kBufs], off_ys[kBufs], off_rp[kBufs], off_wst[kWTabs], off_offs;
     uint32_t off_zs, off_zbuf, off_uw, off_W1, off_b1, off_w2, off_pidx, off_plog, off_U, off_bar;
     float inv_perq, inv_E, inv_kp;
 };
@@ -174,8 +176,9 @@ __device__ __forceinline__ void tile_next(const PipeParams &P, TileIter &it) {
 }
 
 // ---------------------------------------------------------------- mbarriers
-// Shared words: full[0..1] (stage -> mix), done[0..1] (mix -> stage), zbar
+// Shared words: full[kBufs] (stage -> mix), done[kBufs] (mix -> stage), zbar
 // (unit sums of the next run's example copied into shared memory).
+constexpr uint32_t kFullBar = 0, kDoneBar = 8 * kBufs, kZBar = 16 * kBufs;
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
@@ -226,11 +229,11 @@ __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
     const uint2 *offs = reinterpret_cast<const uint2 *>(sm + P.off_offs);
     uint32_t t = 0, run = 0;
     for (TileIter it{blockIdx.x, 0}; it.q < P.runs; ++t) {
-        const int b = (int)(t & 1u);
-        if (!mbar_wait(bars + 8 * b, (t >> 1) & 1u, P.ctrl, it.q)) break;
+        const int b = (int)(t % kBufs);
+        if (!mbar_wait(bars + kFullBar + 8 * b, (t / kBufs) & 1u, P.ctrl, it.q)) break;
         const unsigned char *xs = sm + P.off_xs[b];
         uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[b]);
-        const float2 *wts = reinterpret_cast<const float2 *>(sm + P.off_wst[run % 3]);
+        const float2 *wts = reinterpret_cast<const float2 *>(sm + P.off_wst[run % kWTabs]);
         // expert pairs: warp w's groups take pairs w + 8h of each block of 32,
         // so the groups' output stores and table reads hit different banks
         for (int blk = 0; blk < NP; blk += kMixWarps * kGPW) {
@@ -285,7 +288,7 @@ __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
         }
         // the output tile may leave through the async proxy (bulk copy)
         if (P.bulk_y) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        mbar_arrive(bars + 16 + 8 * b);
+        mbar_arrive(bars + kDoneBar + 8 * b);
         const uint32_t q0 = it.q;
         tile_next(P, it);
         run += it.q != q0;
@@ -297,33 +300,58 @@ __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
 // eight channels) that become eight words of the transposed tile
 // (stage_x_tile's layout); units are numbered so that a warp's stores are
 // conflict-free, and thread st takes units st + kStageT * r.
-__device__ __forceinline__ void stage_load(const PipeParams &P, const TileRef &tr, int st, uint4 *v) {
+// A stage thread's units, fixed for the whole launch: position pa of the low
+// half (pb = pa + kGS), element offset of the loads in a tile of x, byte
+// offset of the stores in a tile buffer (-1: no unit).
+struct StageUnits {
+    int pa[kStageU], src[kStageU], dst[kStageU];
+};
+
+__device__ __forceinline__ StageUnits stage_units(const PipeParams &P, int st) {
+    StageUnits su;
     const int CC = P.C >> 3, per_q = 4 * ((CC + 7) & ~7), units = kGS * per_q;
-    const uint16_t *xt = P.x + ((size_t)tr.n * P.HW + tr.p0) * P.C;
 #pragma unroll
     for (int r = 0; r < kStageU; ++r) {
         const int u = st + r * kStageT;
         int q, j, cc;
         stage_unit_coords(u, per_q, P.inv_perq, q, j, cc);
-        const int pa = q + 2 * kGS * j, pb = pa + kGS;
         const bool ok = u < units && cc < CC;
-        v[2 * r] = ok && pa < tr.np ? __ldcs(reinterpret_cast<const uint4 *>(xt + (size_t)pa * P.C + cc * 8))
+        su.pa[r] = ok ? q + 2 * kGS * j : kTP;
+        su.src[r] = su.pa[r] * P.C + cc * 8;
+        su.dst[r] = ok ? (cc * 8) * kRB + (((q ^ (cc & kFM)) << 4) | (j << 2)) : -1;
+    }
+    return su;
+}
+
+__device__ __forceinline__ void stage_load(const PipeParams &P, const TileRef &tr,
+                                           const StageUnits &su, uint4 *v) {
+    const uint16_t *xt = P.x + ((size_t)tr.n * P.HW + tr.p0) * P.C;
+#pragma unroll
+    for (int r = 0; r < kStageU; ++r) {
+        v[2 * r] = su.pa[r] < tr.np ? __ldcs(reinterpret_cast<const uint4 *>(xt + su.src[r]))
                                     : make_uint4(0u, 0u, 0u, 0u);
-        v[2 * r + 1] = ok && pb < tr.np
-                           ? __ldcs(reinterpret_cast<const uint4 *>(xt + (size_t)pb * P.C + cc * 8))
+        v[2 * r + 1] = su.pa[r] + kGS < tr.np
+                           ? __ldcs(reinterpret_cast<const uint4 *>(xt + su.src[r] + kGS * P.C))
                            : make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
-__device__ __forceinline__ void stage_store(const PipeParams &P, unsigned char *xs, int st,
+// Eight words of the transposed tile per unit (layout of stage_x_tile).
+__device__ __forceinline__ void stage_store(unsigned char *xs, const StageUnits &su,
                                             const uint4 *v) {
-    const int CC = P.C >> 3, per_q = 4 * ((CC + 7) & ~7), units = kGS * per_q;
 #pragma unroll
     for (int r = 0; r < kStageU; ++r) {
-        const int u = st + r * kStageT;
-        int q, j, cc;
-        stage_unit_coords(u, per_q, P.inv_perq, q, j, cc);
-        if (u < units && cc < CC) store_unit<kGS>(xs, q, j, cc, v[2 * r], v[2 * r + 1]);
+        if (su.dst[r] < 0) continue;
+        unsigned char *d = xs + su.dst[r];
+        const uint4 va = v[2 * r], vb = v[2 * r + 1];
+        *reinterpret_cast<uint32_t *>(d + 0 * kRB) = __byte_perm(va.x, vb.x, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 1 * kRB) = __byte_perm(va.x, vb.x, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 2 * kRB) = __byte_perm(va.y, vb.y, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 3 * kRB) = __byte_perm(va.y, vb.y, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 4 * kRB) = __byte_perm(va.z, vb.z, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 5 * kRB) = __byte_perm(va.z, vb.z, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 6 * kRB) = __byte_perm(va.w, vb.w, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 7 * kRB) = __byte_perm(va.w, vb.w, 0x7632);
     }
 }
 
@@ -332,9 +360,9 @@ __device__ __forceinline__ void stage_store(const PipeParams &P, unsigned char *
 // sums of example n (in unit order, one channel per thread) and evaluates the
 // gate of every expert: u = z at the support in deployment order,
 // h = ReLU(W1 u + b1), g = w2 . h + b2, tau (Eq. (tau)), a = softmax(L / tau)
-// (Eq. (weights)). The weights go to one of three weight tables in shared
+// (Eq. (weights)). The weights go to one of kWTabs weight tables in shared
 // memory (pslot layout; runs use them in turn, so the mix role may still read
-// the two previous runs' tables). Every CTA
+// the kBufs previous runs' tables). Every CTA
 // with a run of example n evaluates the same gate from the same z (identical
 // results); the CTA with the example's first run also writes z and tau to the
 // workspace.
@@ -432,7 +460,7 @@ __device__ __forceinline__ void zsum_prefetch(const PipeParams &P, unsigned char
     asm volatile(
         "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, [%0];"
-        ::"r"(smem_u32(sm + P.off_bar) + 32), "r"(bytes), "r"(smem_u32(sm + P.off_zbuf)), "l"(src)
+        ::"r"(smem_u32(sm + P.off_bar) + kZBar), "r"(bytes), "r"(smem_u32(sm + P.off_zbuf)), "l"(src)
         : "memory");
 }
 
@@ -445,7 +473,7 @@ __device__ bool stage_gate(const PipeParams &P, unsigned char *sm, int n, bool o
     const int st = threadIdx.x - kMixT;
     float *zs = reinterpret_cast<float *>(sm + P.off_zs);
     const unsigned long long *zb = reinterpret_cast<const unsigned long long *>(sm + P.off_zbuf);
-    bool ok = mbar_wait(smem_u32(sm + P.off_bar) + 32, zph, P.ctrl, item);
+    bool ok = mbar_wait(smem_u32(sm + P.off_bar) + kZBar, zph, P.ctrl, item);
     for (int c = st; c < P.C && ok; c += kStageT) {
         const unsigned long long *pc = P.part + (size_t)n * P.S * P.C + c;
         unsigned long long v[kMaxUnits];
@@ -561,8 +589,9 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
     const int st = threadIdx.x - kMixT;
     const uint32_t bars = smem_u32(sm + P.off_bar);
     uint4 pre[2 * kStageU];
+    const StageUnits su = stage_units(P, st);
     TileIter it{blockIdx.x, 0};
-    TileRef prev[2] = {{0, 0, 0}, {0, 0, 0}};  // tiles held by the two buffers
+    TileRef prev[kBufs];  // tiles held by the buffers
     uint32_t t = 0, run = 0;
     uint32_t zissued = 0;  // unit-sum copies started (run r's copy is phase r of zbar)
     bool alive = true;
@@ -577,32 +606,33 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
             if (st == 0) zsum_prefetch(P, sm, (int)((it.q + gridDim.x) / (uint32_t)P.RN));
             zissued = 2;
         }
-        stage_load(P, tr, st, pre);
+        stage_load(P, tr, su, pre);
     }
     for (; alive && it.q < P.runs; ++t) {
-        const int b = (int)(t & 1u);
+        const int b = (int)(t % kBufs);
         const TileRef tr = tile_of(P, it);
-        if (t >= 2) {
-            // buffer b held tile t - 2: once mixed, write it out
-            const bool ok = mbar_wait(bars + 16 + 8 * b, ((t - 2) >> 1) & 1u, P.ctrl, it.q);
+        if (t >= kBufs) {
+            // buffer b held tile t - kBufs: once mixed, write it out
+            const bool ok =
+                mbar_wait(bars + kDoneBar + 8 * b, ((t - kBufs) / kBufs) & 1u, P.ctrl, it.q);
             if (!bar_and(kBarStage, kStageT, ok)) { alive = false; break; }
             copy_tile(P, sm, b, prev[b], st);
         }
         prev[b] = tr;
-        stage_store(P, sm + P.off_xs[b], st, pre);
-        // the bulk copy of tile t - 2 has read ys[b] before mix may overwrite it
+        stage_store(sm + P.off_xs[b], su, pre);
+        // the bulk copy of tile t - kBufs has read ys[b] before mix may overwrite it
         if (P.bulk_y && st == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-        mbar_arrive(bars + 8 * b);
+        mbar_arrive(bars + kFullBar + 8 * b);
         const uint32_t q0 = it.q;
         tile_next(P, it);
         if (it.q < P.runs) {
             const TileRef nt = tile_of(P, it);
             // a new run: its gate first (no prefetched data live across it), into
-            // the weight table that the mix role's last two runs do not use
+            // a weight table that none of the runs still in the buffers use
             if (it.q != q0) {
                 ++run;
                 if (!stage_gate(P, sm, nt.n, it.q % (uint32_t)P.RN == 0, ready, it.q,
-                                reinterpret_cast<float *>(sm + P.off_wst[run % 3]), run & 1u)) {
+                                reinterpret_cast<float *>(sm + P.off_wst[run % kWTabs]), run & 1u)) {
                     alive = false;
                     break;
                 }
@@ -611,14 +641,14 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
                     zissued = run + 2;
                 }
             }
-            stage_load(P, nt, st, pre);
+            stage_load(P, nt, su, pre);
         }
     }
     if (alive) {
-        // the last two tiles
-        for (uint32_t tt = t >= 2 ? t - 2 : 0; tt < t; ++tt) {
-            const int b = (int)(tt & 1u);
-            const bool ok = mbar_wait(bars + 16 + 8 * b, (tt >> 1) & 1u, P.ctrl, blockIdx.x);
+        // the last tiles
+        for (uint32_t tt = t >= kBufs ? t - kBufs : 0; tt < t; ++tt) {
+            const int b = (int)(tt % kBufs);
+            const bool ok = mbar_wait(bars + kDoneBar + 8 * b, (tt / kBufs) & 1u, P.ctrl, blockIdx.x);
             if (!bar_and(kBarStage, kStageT, ok)) break;
             copy_tile(P, sm, b, prev[b], st);
         }
@@ -628,7 +658,7 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
     if (st == 0) {
         if (P.bulk_y) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
         if (!alive && zissued > 0) {
-            const uint32_t zb = smem_u32(sm + P.off_bar) + 32;
+            const uint32_t zb = smem_u32(sm + P.off_bar) + kZBar;
             for (uint32_t i = 0; i < kSpinLimit && !mbar_test(zb, (zissued - 1) & 1u); ++i)
                 __nanosleep(256);
         }
@@ -784,7 +814,7 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
                 reinterpret_cast<float *>(sm + P.off_plog)[q] = __ldg(P.plog + q);
             }
         }
-        for (int q = threadIdx.x; q < 2 * (kRB / 4); q += kMixT + kStageT) {
+        for (int q = threadIdx.x; q < kBufs * (kRB / 4); q += kMixT + kStageT) {
             const int b = q / (kRB / 4), w = q - b * (kRB / 4);
             reinterpret_cast<uint32_t *>(sm + P.off_xs[b] + (size_t)P.C * kRB)[w] = 0u;
         }
@@ -797,15 +827,15 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
             }
             const int sl = 2 * pslot(el, P.kp, i >> 1) + (i & 1);
             reinterpret_cast<uint32_t *>(sm + P.off_offs)[sl] = off;
-            for (int b = 0; b < 3; ++b) reinterpret_cast<float *>(sm + P.off_wst[b])[sl] = 0.f;
+            for (int b = 0; b < kWTabs; ++b) reinterpret_cast<float *>(sm + P.off_wst[b])[sl] = 0.f;
         }
         if (threadIdx.x == 0) {
             const uint32_t bars = smem_u32(sm + P.off_bar);
-            mbar_init(bars + 0, kStageT);
-            mbar_init(bars + 8, kStageT);
-            mbar_init(bars + 16, kMixT);
-            mbar_init(bars + 24, kMixT);
-            mbar_init(bars + 32, 1);
+            for (int b = 0; b < kBufs; ++b) {
+                mbar_init(bars + kFullBar + 8 * b, kStageT);
+                mbar_init(bars + kDoneBar + 8 * b, kMixT);
+            }
+            mbar_init(bars + kZBar, 1);
             // zbar completes through the async proxy (bulk copies)
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
@@ -831,14 +861,16 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
 struct PipePlan {
     int kp = 0, Es = 0, ks = 0, Kg = 0;
     bool gate_tabs = false;
-    size_t off_xs[2] = {}, off_ys[2] = {}, off_rp[2] = {}, off_wst[3] = {}, off_offs = 0;
+    size_t off_xs[kBufs] = {}, off_ys[kBufs] = {}, off_rp[kBufs] = {}, off_wst[kWTabs] = {};
+    size_t off_offs = 0;
     size_t off_zs = 0, off_zbuf = 0, off_uw = 0, off_W1 = 0, off_b1 = 0, off_w2 = 0;
     size_t off_pidx = 0, off_plog = 0, off_U = 0, off_bar = 0, smem = 0;
 };
 
-// Shared memory: two x buffers of C + 1 rows (row C = zeros), two output
-// tiles, two residual partial blocks, the row-offset table, three weight
-// tables, the gate's z, the gate parameters, [support tables,] U, mbarriers.
+// Shared memory: kBufs x buffers of C + 1 rows (row C = zeros), kBufs output
+// tiles and residual partial blocks, the row-offset table, kWTabs weight
+// tables, the gate's z and unit-sum copy, the gate parameters, [support
+// tables,] U, mbarriers.
 bool pipe_plan(int C, int R, int k, PipePlan *plan) {
     // C <= 256: every staging unit of a tile has its thread (kStageU per thread)
     if (C % 8 != 0 || C < 8 || C > 256 || k < 1 || k > kGateMaxK || R < 1) return false;
@@ -854,11 +886,11 @@ bool pipe_plan(int C, int R, int k, PipePlan *plan) {
         off += bytes;
         return o;
     };
-    for (int b = 0; b < 2; ++b) p.off_xs[b] = take((size_t)(C + 1) * kRB, 128);
-    for (int b = 0; b < 2; ++b) p.off_ys[b] = take((size_t)kTP * p.Es * 2, 16);
-    for (int b = 0; b < 2; ++b) p.off_rp[b] = take((size_t)kGroups * kRPS * 4, 16);
+    for (int b = 0; b < kBufs; ++b) p.off_xs[b] = take((size_t)(C + 1) * kRB, 128);
+    for (int b = 0; b < kBufs; ++b) p.off_ys[b] = take((size_t)kTP * p.Es * 2, 16);
+    for (int b = 0; b < kBufs; ++b) p.off_rp[b] = take((size_t)kGroups * kRPS * 4, 16);
     p.off_offs = take((size_t)pslot_count(R, p.kp) * 8, 16);
-    for (int b = 0; b < 3; ++b) p.off_wst[b] = take((size_t)pslot_count(R, p.kp) * 8, 16);
+    for (int b = 0; b < kWTabs; ++b) p.off_wst[b] = take((size_t)pslot_count(R, p.kp) * 8, 16);
     p.off_zs = take((size_t)C * 4, 16);
     p.off_zbuf = take((size_t)kMaxUnits * C * 8, 128);
     p.off_uw = take((size_t)(kStageT / 32) * k * 4, 16);
@@ -872,7 +904,7 @@ bool pipe_plan(int C, int R, int k, PipePlan *plan) {
         p.off_plog = take((size_t)R * k * 4, 16);
     }
     p.off_U = take((size_t)C * 4, 16);
-    p.off_bar = take(40, 8);
+    p.off_bar = take(16 * kBufs + 8, 8);
     p.smem = off;
     if (p.smem > 227 * 1024) return false;
     *plan = p;
@@ -961,14 +993,14 @@ cudaError_t launch_pipe(const uint16_t *x, int N, int HW, int C, int R, int k,
     P.bulk_y = ((long long)HW * (R + 1)) % 8 == 0 && (reinterpret_cast<uintptr_t>(y) & 15u) == 0;
     if (P.bulk_y) P.Es = R + 1;
     P.gate_tabs = plan.gate_tabs ? 1 : 0;
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kBufs; ++b) {
         P.off_xs[b] = (uint32_t)plan.off_xs[b];
         P.off_ys[b] = (uint32_t)plan.off_ys[b];
         P.off_rp[b] = (uint32_t)plan.off_rp[b];
     }
     P.off_zs = (uint32_t)plan.off_zs;
     P.off_zbuf = (uint32_t)plan.off_zbuf;
-    for (int b = 0; b < 3; ++b) P.off_wst[b] = (uint32_t)plan.off_wst[b];
+    for (int b = 0; b < kWTabs; ++b) P.off_wst[b] = (uint32_t)plan.off_wst[b];
     P.off_offs = (uint32_t)plan.off_offs;
     P.off_uw = (uint32_t)plan.off_uw;
     P.off_W1 = (uint32_t)plan.off_W1;
