@@ -200,11 +200,22 @@ __device__ __forceinline__ bool mbar_test(uint32_t a, uint32_t parity) {
     return ok != 0;
 }
 // Bounded wait for the phase with the given parity to complete.
+// try_wait suspends the warp in hardware (up to the hint) instead of
+// spinning, so waiting warps leave the issue slots to the other roles.
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(a), "r"(parity), "r"(1000u)
+        : "memory");
+    return ok != 0;
+}
 __device__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t *ctrl, uint32_t item) {
     for (uint32_t it = 0; it < kSpinLimit; ++it) {
-        if (mbar_test(a, parity)) return true;
+        if (mbar_try(a, parity)) return true;
         if ((it & 15u) == 15u && ld_relaxed(ctrl + kCtrlError) != 0u) return false;
-        if (it >= 64) __nanosleep(128);
     }
     report_timeout(ctrl, item);
     return false;
