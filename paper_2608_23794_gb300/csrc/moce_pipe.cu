@@ -54,7 +54,7 @@ constexpr int kGroups = kMixT / kGS;  // mixing groups per CTA
 constexpr int kRPS = kTP + 8;         // row stride (floats) of the residual partial sums
 constexpr int kBarStage = 2, kBarPrologue = 3;
 constexpr int kBufs = 2;              // tile buffers (x, y, residual sums) between stage and mix
-constexpr int kWTabs = kBufs + 1;     // per-run weight tables: the mix role may read kBufs runs
+constexpr int kWTabs = kBufs + 1;     // run tables: the mix role may still read kBufs runs
 constexpr int kStageU = 4;            // staging units (2 x 16 bytes) per stage thread and tile
 constexpr int kRun = 7;               // mixing tiles per run (one gate per run)
 constexpr int kPoolWin = 6;           // rolling window of 16-byte loads per pool thread
@@ -86,7 +86,7 @@ struct PipeParams {
     int cpw, rpi;                 // pool: 8-channel blocks per warp, rows per load instruction
     int kp, Es, ks, Kg, gate_tabs;  // Kg: padded gate width of the group gate, 0: warp gate
     int bulk_y;                   // output tiles leave by one bulk copy (rows of E = R + 1)
-    uint32_t off_xs[kBufs], off_ys[kBufs], off_rp[kBufs], off_wst[kWTabs], off_offs;
+    uint32_t off_xs[kBufs], off_ys[kBufs], off_rp[kBufs], off_tab[kWTabs];
     uint32_t off_zs, off_zbuf, off_uw, off_W1, off_b1, off_w2, off_pidx, off_plog, off_U, off_bar;
     float inv_perq, inv_E, inv_kp;
 };
@@ -100,51 +100,14 @@ template <int N> __device__ __forceinline__ void set_role_regs() {
         asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
 }
 
-// Slot (8-byte units) of entries (2*i2, 2*i2+1) of expert el in the offset
-// table (uint2: two row offsets) and in the weight tables (float2): the four
-// groups of a warp mix experts 16 apart, so block b of 16 experts is shifted
-// by b slots and their reads hit different banks.
+// Slot (uint4 units) of entries (2*i2, 2*i2+1) of expert el in a run table
+// {row offset, row offset, weight, weight}: the four groups of a warp mix
+// experts 16 apart, so block b of 16 experts is shifted by b slots and their
+// reads hit different banks.
 __device__ __forceinline__ int pslot(int el, int kp, int i2) {
     return el * (kp >> 1) + (el >> 4) + i2;
 }
 inline int pslot_count(int R, int kp) { return (R - 1) * (kp >> 1) + ((R - 1) >> 4) + (kp >> 1); }
-
-// Weighted sums of two experts' entry pairs for the lane's 8 positions; each
-// step reads the row offsets and the weights of two support positions per
-// expert, then one 16-byte chunk of each row.
-__device__ __forceinline__ void mix_pairs2(const unsigned char *xs, const uint2 *oa, const uint2 *ob,
-                                           const float2 *wa, const float2 *wb, int npairs,
-                                           uint32_t lx, float2 &a0, float2 &a1, float2 &a2,
-                                           float2 &a3, float2 &b0, float2 &b1, float2 &b2,
-                                           float2 &b3) {
-#pragma unroll 2
-    for (int i2 = 0; i2 < npairs; ++i2) {
-        const uint2 ra = oa[i2], rb = ob[i2];
-        const float2 ga = wa[i2], gb = wb[i2];
-        const uint4 va0 = lds128(xs + (ra.x ^ lx));
-        const uint4 va1 = lds128(xs + (ra.y ^ lx));
-        const uint4 vb0 = lds128(xs + (rb.x ^ lx));
-        const uint4 vb1 = lds128(xs + (rb.y ^ lx));
-        const float2 wa0 = make_float2(ga.x, ga.x), wa1 = make_float2(ga.y, ga.y);
-        const float2 wb0 = make_float2(gb.x, gb.x), wb1 = make_float2(gb.y, gb.y);
-        a0 = __ffma2_rn(wa0, unpack2(va0.x), a0);
-        a1 = __ffma2_rn(wa0, unpack2(va0.y), a1);
-        a2 = __ffma2_rn(wa0, unpack2(va0.z), a2);
-        a3 = __ffma2_rn(wa0, unpack2(va0.w), a3);
-        b0 = __ffma2_rn(wb0, unpack2(vb0.x), b0);
-        b1 = __ffma2_rn(wb0, unpack2(vb0.y), b1);
-        b2 = __ffma2_rn(wb0, unpack2(vb0.z), b2);
-        b3 = __ffma2_rn(wb0, unpack2(vb0.w), b3);
-        a0 = __ffma2_rn(wa1, unpack2(va1.x), a0);
-        a1 = __ffma2_rn(wa1, unpack2(va1.y), a1);
-        a2 = __ffma2_rn(wa1, unpack2(va1.z), a2);
-        a3 = __ffma2_rn(wa1, unpack2(va1.w), a3);
-        b0 = __ffma2_rn(wb1, unpack2(vb1.x), b0);
-        b1 = __ffma2_rn(wb1, unpack2(vb1.y), b1);
-        b2 = __ffma2_rn(wb1, unpack2(vb1.z), b2);
-        b3 = __ffma2_rn(wb1, unpack2(vb1.w), b3);
-    }
-}
 
 // This CTA's mixing tiles, in order: runs q = blockIdx.x, blockIdx.x + G, ...
 // of up to kRun consecutive tiles of one example.
@@ -237,14 +200,13 @@ __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
     const int R = P.R, kp = P.kp, NP = (R + 1) >> 1, Es = P.Es;
     const int32_t *s_resid = reinterpret_cast<const int32_t *>(sm + P.off_U);
     const uint32_t bars = smem_u32(sm + P.off_bar);
-    const uint2 *offs = reinterpret_cast<const uint2 *>(sm + P.off_offs);
     uint32_t t = 0, run = 0;
     for (TileIter it{blockIdx.x, 0}; it.q < P.runs; ++t) {
         const int b = (int)(t % kBufs);
         if (!mbar_wait(bars + kFullBar + 8 * b, (t / kBufs) & 1u, P.ctrl, it.q)) break;
         const unsigned char *xs = sm + P.off_xs[b];
         uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[b]);
-        const float2 *wts = reinterpret_cast<const float2 *>(sm + P.off_wst[run % kWTabs]);
+        const uint4 *tab = reinterpret_cast<const uint4 *>(sm + P.off_tab[run % kWTabs]);
         // expert pairs: warp w's groups take pairs w + 8h of each block of 32,
         // so the groups' output stores and table reads hit different banks
         for (int blk = 0; blk < NP; blk += kMixWarps * kGPW) {
@@ -255,8 +217,8 @@ __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
             float2 b0 = a0, b1 = a0, b2 = a0, b3 = a0;
             // an odd last expert pairs with itself; its twin's result is dropped
             const int ebb = eb < R ? eb : ea;
-            mix_pairs2(xs, offs + pslot(ea, kp, 0), offs + pslot(ebb, kp, 0), wts + pslot(ea, kp, 0),
-                       wts + pslot(ebb, kp, 0), kp >> 1, lx, a0, a1, a2, a3, b0, b1, b2, b3);
+            mix_entries2(xs, tab + pslot(ea, kp, 0), tab + pslot(ebb, kp, 0), kp >> 1, lx, a0, a1,
+                         a2, a3, b0, b1, b2, b3);
             // lane lig's positions are lig + 8 m, m = 0..7
             if (P.bulk_y) {
                 // rows of odd length: 16-bit stores
@@ -371,8 +333,8 @@ __device__ __forceinline__ void stage_store(unsigned char *xs, const StageUnits 
 // sums of example n (in unit order, one channel per thread) and evaluates the
 // gate of every expert: u = z at the support in deployment order,
 // h = ReLU(W1 u + b1), g = w2 . h + b2, tau (Eq. (tau)), a = softmax(L / tau)
-// (Eq. (weights)). The weights go to one of kWTabs weight tables in shared
-// memory (pslot layout; runs use them in turn, so the mix role may still read
+// (Eq. (weights)). The weights go to the weight fields of one of kWTabs run
+// tables (pslot layout; runs use them in turn, so the mix role may still read
 // the kBufs previous runs' tables). Every CTA
 // with a run of example n evaluates the same gate from the same z (identical
 // results); the CTA with the example's first run also writes z and tau to the
@@ -385,6 +347,8 @@ __device__ __forceinline__ void stage_store(unsigned char *xs, const StageUnits 
 template <int K>
 __device__ __forceinline__ void gate_groups(const PipeParams &P, const unsigned char *sm,
                                             const float *zs, float *ws_w, int n, bool out) {
+    constexpr int kE = 2;                  // experts per group at a time (independent chains)
+    constexpr int kNG = kStageT / K;       // groups
     const int st = threadIdx.x - kMixT;
     const int k = P.k, kp = P.kp;
     const int j = st & (K - 1), gi = st / K;
@@ -395,33 +359,56 @@ __device__ __forceinline__ void gate_groups(const PipeParams &P, const unsigned 
     const float *plog = P.gate_tabs ? reinterpret_cast<const float *>(sm + P.off_plog) : P.plog;
     const float b2 = __ldg(P.b2);
     const bool pos = j < k;
-    // lane j's row of W1 (hidden unit j), b1 and w2 stay in registers
+    // lane j's row of W1 (hidden unit j), b1 and w2 stay in registers; row
+    // element (i + j) mod K is read at step i, so the lanes hit different banks
     float wr[K];
 #pragma unroll
     for (int i = 0; i < K; ++i) wr[i] = W1p[j * K + ((i + j) & (K - 1))];
     const float b1j = b1p[j], w2j = w2p[j];
-    // two experts per group at a time: their latency chains overlap
-#pragma unroll 2
-    for (int e0 = 0; e0 < P.R; e0 += kStageT / K) {
-        const int e = e0 + gi;
-        const bool act = e < P.R && pos;
-        const float uj = act ? zs[pidx[(size_t)e * k + j]] : 0.f;
-        float h = b1j;
+    for (int e0 = 0; e0 < P.R; e0 += kE * kNG) {
+        int e[kE];
+        bool act[kE];
+        float uj[kE], h[kE];
 #pragma unroll
-        for (int i = 0; i < K; ++i)
-            h = fmaf(wr[i], __shfl_sync(0xffffffffu, uj, (i + j) & (K - 1), K), h);
-        float gp = w2j * fmaxf(h, 0.f);
+        for (int c = 0; c < kE; ++c) {
+            e[c] = e0 + gi + c * kNG;
+            act[c] = e[c] < P.R && pos;
+            uj[c] = act[c] ? zs[pidx[(size_t)e[c] * k + j]] : 0.f;
+            h[c] = b1j;
+        }
 #pragma unroll
-        for (int o = K / 2; o > 0; o >>= 1) gp += __shfl_xor_sync(0xffffffffu, gp, o, K);
-        const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-(gp + b2)));
-        const float L = act ? plog[(size_t)e * k + j] : 0.f;
-        const float L0 = __shfl_sync(0xffffffffu, L, 0, K);  // position 0 holds the largest logit
-        const float ex = act ? expf((L - L0) / tau) : 0.f;
-        float zsum = ex;
+        for (int i = 0; i < K; ++i) {
+            const int src = (i + j) & (K - 1);
 #pragma unroll
-        for (int o = K / 2; o > 0; o >>= 1) zsum += __shfl_xor_sync(0xffffffffu, zsum, o, K);
-        if (act) ws_w[2 * pslot(e, kp, j >> 1) + (j & 1)] = ex / zsum;
-        if (out && act && j == 0) P.tau[(size_t)n * P.R + e] = tau;
+            for (int c = 0; c < kE; ++c)
+                h[c] = fmaf(wr[i], __shfl_sync(0xffffffffu, uj[c], src, K), h[c]);
+        }
+        float gp[kE], L[kE];
+#pragma unroll
+        for (int c = 0; c < kE; ++c) {
+            gp[c] = w2j * fmaxf(h[c], 0.f);
+            L[c] = act[c] ? plog[(size_t)e[c] * k + j] : 0.f;
+        }
+#pragma unroll
+        for (int o = K / 2; o > 0; o >>= 1)
+#pragma unroll
+            for (int c = 0; c < kE; ++c) gp[c] += __shfl_xor_sync(0xffffffffu, gp[c], o, K);
+        float ex[kE], zsum[kE];
+#pragma unroll
+        for (int c = 0; c < kE; ++c) {
+            const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-(gp[c] + b2)));
+            const float L0 = __shfl_sync(0xffffffffu, L[c], 0, K);  // position 0: largest logit
+            ex[c] = act[c] ? expf((L[c] - L0) / tau) : 0.f;
+            zsum[c] = ex[c];
+            if (out && act[c] && j == 0) P.tau[(size_t)n * P.R + e[c]] = tau;
+        }
+#pragma unroll
+        for (int o = K / 2; o > 0; o >>= 1)
+#pragma unroll
+            for (int c = 0; c < kE; ++c) zsum[c] += __shfl_xor_sync(0xffffffffu, zsum[c], o, K);
+#pragma unroll
+        for (int c = 0; c < kE; ++c)
+            if (act[c]) ws_w[4 * pslot(e[c], kp, j >> 1) + 2 + (j & 1)] = ex[c] / zsum[c];
     }
 }
 
@@ -456,8 +443,8 @@ __device__ void gate_warps(const PipeParams &P, unsigned char *sm, const float *
         const float ex0 = lane < k ? expf((L[lane] - L0) / tau) : 0.f;
         const float ex1 = lane + 32 < k ? expf((L[lane + 32] - L0) / tau) : 0.f;
         const float zsum = warp_sum(ex0 + ex1);
-        if (lane < k) ws_w[2 * pslot(e, kp, lane >> 1) + (lane & 1)] = ex0 / zsum;
-        if (lane + 32 < k) ws_w[2 * pslot(e, kp, (lane + 32) >> 1) + (lane & 1)] = ex1 / zsum;
+        if (lane < k) ws_w[4 * pslot(e, kp, lane >> 1) + 2 + (lane & 1)] = ex0 / zsum;
+        if (lane + 32 < k) ws_w[4 * pslot(e, kp, (lane + 32) >> 1) + 2 + (lane & 1)] = ex1 / zsum;
         if (out && lane == 0) P.tau[(size_t)n * P.R + e] = tau;
         __syncwarp();
     }
@@ -611,7 +598,7 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
         if (st == 0) zsum_prefetch(P, sm, tr.n);
         zissued = 1;
         alive = stage_gate(P, sm, tr.n, it.q % (uint32_t)P.RN == 0, ready, it.q,
-                           reinterpret_cast<float *>(sm + P.off_wst[0]), 0u);
+                           reinterpret_cast<float *>(sm + P.off_tab[0]), 0u);
         // the unit sums of the next run's example arrive while this run is mixed
         if (alive && it.q + gridDim.x < P.runs) {
             if (st == 0) zsum_prefetch(P, sm, (int)((it.q + gridDim.x) / (uint32_t)P.RN));
@@ -639,11 +626,11 @@ __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t read
         if (it.q < P.runs) {
             const TileRef nt = tile_of(P, it);
             // a new run: its gate first (no prefetched data live across it), into
-            // a weight table that none of the runs still in the buffers use
+            // a run table that none of the runs still in the buffers use
             if (it.q != q0) {
                 ++run;
                 if (!stage_gate(P, sm, nt.n, it.q % (uint32_t)P.RN == 0, ready, it.q,
-                                reinterpret_cast<float *>(sm + P.off_wst[run % kWTabs]), run & 1u)) {
+                                reinterpret_cast<float *>(sm + P.off_tab[run % kWTabs]), run & 1u)) {
                     alive = false;
                     break;
                 }
@@ -794,7 +781,7 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
     } else {
         // data that stays for the whole launch (mix and stage roles): U list,
         // gate parameters and support tables, the zero row of both x buffers,
-        // the row-offset table and zeroed weight tables
+        // the run tables' row offsets (weights start at zero)
         int32_t *s_resid = reinterpret_cast<int32_t *>(sm + P.off_U);
         for (int i = threadIdx.x; i < P.nU; i += kMixT + kStageT) s_resid[i] = __ldg(P.resid + i);
         float *W1s = reinterpret_cast<float *>(sm + P.off_W1);
@@ -836,9 +823,12 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
                 const uint32_t c = (uint32_t)__ldg(P.pidx + (size_t)el * P.k + i);
                 off = (c * kRB) | (((c >> 3) & kFM) << 4);
             }
-            const int sl = 2 * pslot(el, P.kp, i >> 1) + (i & 1);
-            reinterpret_cast<uint32_t *>(sm + P.off_offs)[sl] = off;
-            for (int b = 0; b < kWTabs; ++b) reinterpret_cast<float *>(sm + P.off_wst[b])[sl] = 0.f;
+            for (int b = 0; b < kWTabs; ++b) {
+                uint32_t *w = reinterpret_cast<uint32_t *>(
+                    reinterpret_cast<uint4 *>(sm + P.off_tab[b]) + pslot(el, P.kp, i >> 1));
+                w[i & 1] = off;
+                w[2 + (i & 1)] = 0u;
+            }
         }
         if (threadIdx.x == 0) {
             const uint32_t bars = smem_u32(sm + P.off_bar);
@@ -872,15 +862,13 @@ __global__ void __launch_bounds__(kPipeT, 1) moce_pipe_kernel(const PipeParams P
 struct PipePlan {
     int kp = 0, Es = 0, ks = 0, Kg = 0;
     bool gate_tabs = false;
-    size_t off_xs[kBufs] = {}, off_ys[kBufs] = {}, off_rp[kBufs] = {}, off_wst[kWTabs] = {};
-    size_t off_offs = 0;
+    size_t off_xs[kBufs] = {}, off_ys[kBufs] = {}, off_rp[kBufs] = {}, off_tab[kWTabs] = {};
     size_t off_zs = 0, off_zbuf = 0, off_uw = 0, off_W1 = 0, off_b1 = 0, off_w2 = 0;
     size_t off_pidx = 0, off_plog = 0, off_U = 0, off_bar = 0, smem = 0;
 };
 
 // Shared memory: kBufs x buffers of C + 1 rows (row C = zeros), kBufs output
-// tiles and residual partial blocks, the row-offset table, kWTabs weight
-// tables, the gate's z and unit-sum copy, the gate parameters, [support
+// tiles and residual partial blocks, kWTabs run tables, the gate's z and unit-sum copy, the gate parameters, [support
 // tables,] U, mbarriers.
 bool pipe_plan(int C, int R, int k, PipePlan *plan) {
     // C <= 256: every staging unit of a tile has its thread (kStageU per thread)
@@ -900,8 +888,7 @@ bool pipe_plan(int C, int R, int k, PipePlan *plan) {
     for (int b = 0; b < kBufs; ++b) p.off_xs[b] = take((size_t)(C + 1) * kRB, 128);
     for (int b = 0; b < kBufs; ++b) p.off_ys[b] = take((size_t)kTP * p.Es * 2, 16);
     for (int b = 0; b < kBufs; ++b) p.off_rp[b] = take((size_t)kGroups * kRPS * 4, 16);
-    p.off_offs = take((size_t)pslot_count(R, p.kp) * 8, 16);
-    for (int b = 0; b < kWTabs; ++b) p.off_wst[b] = take((size_t)pslot_count(R, p.kp) * 8, 16);
+    for (int b = 0; b < kWTabs; ++b) p.off_tab[b] = take((size_t)pslot_count(R, p.kp) * 16, 16);
     p.off_zs = take((size_t)C * 4, 16);
     p.off_zbuf = take((size_t)kMaxUnits * C * 8, 128);
     p.off_uw = take((size_t)(kStageT / 32) * k * 4, 16);
@@ -1011,8 +998,7 @@ cudaError_t launch_pipe(const uint16_t *x, int N, int HW, int C, int R, int k,
     }
     P.off_zs = (uint32_t)plan.off_zs;
     P.off_zbuf = (uint32_t)plan.off_zbuf;
-    for (int b = 0; b < kWTabs; ++b) P.off_wst[b] = (uint32_t)plan.off_wst[b];
-    P.off_offs = (uint32_t)plan.off_offs;
+    for (int b = 0; b < kWTabs; ++b) P.off_tab[b] = (uint32_t)plan.off_tab[b];
     P.off_uw = (uint32_t)plan.off_uw;
     P.off_W1 = (uint32_t)plan.off_W1;
     P.off_b1 = (uint32_t)plan.off_b1;
