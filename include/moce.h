@@ -203,6 +203,16 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
                           moce_dtype_t dtype, moce_layout_t layout);
 
 /*
+ * Name of the kernel path moce_forward takes for these arguments:
+ * "moce_pipe_kernel" (the warp-specialised pipeline, NHWC bf16 with
+ * C_in <= 256), "moce_fused_kernel" (the two-group persistent kernel) or
+ * "pool+gate+mix" (one kernel per step). NULL for arguments moce_forward
+ * would reject. Enqueues nothing; the string is static.
+ */
+const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                moce_dtype_t dtype, moce_layout_t layout);
+
+/*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word the
  * forward kernels leave in `ws` (a forward workspace). Returns MOCE_OK,
  * MOCE_ERR_TIMEOUT (a bounded inter-CTA wait gave up; outputs of that call

@@ -187,6 +187,14 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
     return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
 }
 
+const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                moce_dtype_t dtype, moce_layout_t layout) {
+    const int launches = moce_forward_launches(x, N, H, W, C_in, C_out, k, dtype, layout);
+    if (launches == 0) return nullptr;
+    if (launches > 1) return "pool+gate+mix";
+    return pipe_supported(N, H * W, C_in, C_out, k) ? "moce_pipe_kernel" : "moce_fused_kernel";
+}
+
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {
     if (!ws || ws_bytes < kCtrlWords * 4) return MOCE_ERR_INVALID_VALUE;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

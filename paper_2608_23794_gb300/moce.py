@@ -63,6 +63,7 @@ def library():
             "moce_forward": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S, P], I),
             "moce_check_device_error": ([P, S, P], I),
             "moce_forward_launches": ([P, I, I, I, I, I, I, I, I], I),
+            "moce_forward_kernel": ([P, I, I, I, I, I, I, I, I], ctypes.c_char_p),
             "moce_forward_noalloc": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P], I),
         }
         for name, (args, res) in sig.items():
@@ -232,6 +233,15 @@ def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int) -> i
     N, H, W, C = _dims(x, layout)
     return int(library().moce_forward_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
                                                 _LAYOUTS[layout]))
+
+
+def moce_forward_kernel(x: torch.Tensor, layout: str, C_out: int, k: int) -> str:
+    """Name of the kernel path one moce_forward call takes for this input."""
+    N, H, W, C = _dims(x, layout)
+    name = library().moce_forward_kernel(_ptr(x), N, H, W, C, C_out, k, _dtype(x), _LAYOUTS[layout])
+    if name is None:
+        raise MoceError(1, "moce_forward_kernel")
+    return name.decode()
 
 
 def moce_forward_noalloc(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
