@@ -159,6 +159,12 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
                                        b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
                                        s));
     }
+    if (vec && ring_supported(N, HW, C_in, C_out, k)) {
+        return cuda_status(launch_ring(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
+                                       packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
+                                       b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
+                                       s));
+    }
     if (vec && fused_supported(N, HW, C_in, C_out, k)) {
         return cuda_status(launch_fused(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
                                         packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
@@ -182,7 +188,8 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
     if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
         (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
-        (pipe_supported(N, H * W, C_in, C_out, k) || fused_supported(N, H * W, C_in, C_out, k)))
+        (ring_supported(N, H * W, C_in, C_out, k) || pipe_supported(N, H * W, C_in, C_out, k) ||
+         fused_supported(N, H * W, C_in, C_out, k)))
         return 1;
     return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
 }
@@ -192,7 +199,8 @@ const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, in
     const int launches = moce_forward_launches(x, N, H, W, C_in, C_out, k, dtype, layout);
     if (launches == 0) return nullptr;
     if (launches > 1) return "pool+gate+mix";
-    return pipe_supported(N, H * W, C_in, C_out, k) ? "moce_pipe_kernel" : "moce_fused_kernel";
+    if (pipe_supported(N, H * W, C_in, C_out, k)) return "moce_pipe_kernel";
+    return ring_supported(N, H * W, C_in, C_out, k) ? "moce_ring_kernel" : "moce_fused_kernel";
 }
 
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {

@@ -75,6 +75,66 @@ static __device__ bool wait_tagged(const unsigned long long *p, uint32_t tag, un
     return false;
 }
 
+// Sets this warpgroup's registers per thread to N, from the launch's L.
+// The sum over the warpgroups of a launch must stay within threads x L:
+// setmaxnreg.inc waits until the registers are free.
+template <int N, int L> __device__ __forceinline__ void set_role_regs() {
+    static_assert(N % 8 == 0 && N >= 24 && N <= 256, "setmaxnreg count");
+    if constexpr (N > L)
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
+    else if constexpr (N < L)
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
+}
+
+// ---------------------------------------------------------------- mbarriers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+    asm volatile("{\n\t.reg .b64 st;\n\tmbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(a)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint32_t a, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(a), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait for the phase with the given parity to complete.
+// try_wait suspends the warp in hardware (up to the hint) instead of
+// spinning, so waiting warps leave the issue slots to the other roles.
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(a), "r"(parity), "r"(1000u)
+        : "memory");
+    return ok != 0;
+}
+static __device__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t *ctrl, uint32_t item) {
+    for (uint32_t it = 0; it < kSpinLimit; ++it) {
+        if (mbar_try(a, parity)) return true;
+        if ((it & 15u) == 15u && ld_relaxed(ctrl + kCtrlError) != 0u) return false;
+    }
+    report_timeout(ctrl, item);
+    return false;
+}
+
+__device__ __forceinline__ unsigned long long ld_relaxed64(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
 // u / d for 0 <= u < 2^24, 1 <= d and u / d < 2^21, with inv = 1.0f / d: the float
 // estimate is within one of the quotient and is corrected exactly.
 __device__ __forceinline__ int fdiv(int u, int d, float inv) {
@@ -93,6 +153,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return (uint32_t)f32_to_bf16(lo) | ((uint32_t)f32_to_bf16(hi) << 16);
 }
+
 
 // Table slot (uint4 units) of entries (2*i2, 2*i2+1) of expert el. The two
 // lane groups of a warp mix experts 32 apart; block b of 32 experts is shifted

@@ -37,13 +37,31 @@ inline int pool_tile_px(int C) {
     return p2;
 }
 
+// Slot (uint4 units) of entries (2*i2, 2*i2+1) of expert el in a mixing table
+// {row offset, row offset, weight, weight}: the four groups of a warp mix
+// experts 16 apart, so block b of 16 experts is shifted by b slots and their
+// reads hit different banks.
+__host__ __device__ __forceinline__ int pslot(int el, int kp, int i2) {
+    return el * (kp >> 1) + (el >> 4) + i2;
+}
+__host__ __device__ inline int pslot_count(int R, int kp) { return (R - 1) * (kp >> 1) + ((R - 1) >> 4) + (kp >> 1); }
+
+// Positions per tile of the resident-tile kernel (moce_ring.cu).
+constexpr int kRingTile = 64;
+
 struct WsLayout {
     size_t ctrl = 0;      // kCtrlWords uint32
     size_t partial = 0;   // [N][pool_tiles][C] pooling tile sums: fp32 (multi-kernel path) or
-                          // tagged 64-bit words {fp32 bits, epoch + 1} (persistent kernels)
+                          // tagged 64-bit words {fp32 bits, epoch + 1} (persistent kernels);
+                          // [N][ceil(HW/64)][C] fp32 tile sums for the resident-tile kernel
     size_t z = 0;         // [N][C] fp32
     size_t tau = 0;       // [N][R] fp32
-    size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit
+    size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit;
+                          // [N][pslot_count][2] fp32 for the resident-tile kernel
+    size_t zacc = 0;      // [2][N][C] int64 fixed-point channel sums (resident-tile kernel;
+                          // two sets, by the parity of the forward's epoch)
+    size_t sync = 0;      // [2][N] tile arrivals, then [2][N] overflow marks, uint32
+                          // (resident-tile kernel)
     size_t total = 0;
     int pool_px = 0;
     int pool_tiles = 0;
@@ -55,13 +73,18 @@ inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     L.pool_px = pool_tile_px(C);
     L.pool_tiles = (HW + L.pool_px - 1) / L.pool_px;
     L.gate_blocks = (R + kGateExperts - 1) / kGateExperts;
+    const size_t ring_tiles = (size_t)(HW + kRingTile - 1) / kRingTile;
+    const int kp = k + (k & 1);
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+    auto mx = [](size_t a, size_t b) { return a > b ? a : b; };
     L.ctrl = take(kCtrlWords * 4);
-    L.partial = take((size_t)N * L.pool_tiles * C * 8);
+    L.partial = take((size_t)N * mx((size_t)L.pool_tiles * C * 8, ring_tiles * C * 4));
     L.z = take((size_t)N * C * 4);
     L.tau = take((size_t)N * R * 4);
-    L.a = take((size_t)N * R * k * 8);
+    L.a = take((size_t)N * mx((size_t)R * k * 8, (size_t)pslot_count(R, kp) * 8));
+    L.zacc = take((size_t)2 * N * C * 8);
+    L.sync = take((size_t)N * 16);
     L.total = off;
     return L;
 }
@@ -130,5 +153,13 @@ cudaError_t launch_pipe(const uint16_t *x, int N, int HW, int C, int R, int k,
                         cudaStream_t s);
 
 bool pipe_supported(int N, int HW, int C, int R, int k);
+
+cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
+                        const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
+                        const float *W1, const float *b1, const float *w2, const float *b2,
+                        float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
+                        cudaStream_t s);
+
+bool ring_supported(int N, int HW, int C, int R, int k);
 
 }  // namespace moce

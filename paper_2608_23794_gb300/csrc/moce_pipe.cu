@@ -91,23 +91,6 @@ struct PipeParams {
     float inv_perq, inv_E, inv_kp;
 };
 
-// Sets this warpgroup's registers per thread to N (from the launch's count).
-template <int N> __device__ __forceinline__ void set_role_regs() {
-    static_assert(N % 8 == 0 && N >= 24 && N <= 256, "setmaxnreg count");
-    if constexpr (N > kLaunchRegs)
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
-    else if constexpr (N < kLaunchRegs)
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
-}
-
-// Slot (uint4 units) of entries (2*i2, 2*i2+1) of expert el in a run table
-// {row offset, row offset, weight, weight}: the four groups of a warp mix
-// experts 16 apart, so block b of 16 experts is shifted by b slots and their
-// reads hit different banks.
-__device__ __forceinline__ int pslot(int el, int kp, int i2) {
-    return el * (kp >> 1) + (el >> 4) + i2;
-}
-inline int pslot_count(int R, int kp) { return (R - 1) * (kp >> 1) + ((R - 1) >> 4) + (kp >> 1); }
 
 // This CTA's mixing tiles, in order: runs q = blockIdx.x, blockIdx.x + G, ...
 // of up to kRun consecutive tiles of one example.
@@ -142,57 +125,10 @@ __device__ __forceinline__ void tile_next(const PipeParams &P, TileIter &it) {
 // Shared words: full[kBufs] (stage -> mix), done[kBufs] (mix -> stage), zbar
 // (unit sums of the next run's example copied into shared memory).
 constexpr uint32_t kFullBar = 0, kDoneBar = 8 * kBufs, kZBar = 16 * kBufs;
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t a) {
-    asm volatile("{\n\t.reg .b64 st;\n\tmbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(a)
-                 : "memory");
-}
-__device__ __forceinline__ bool mbar_test(uint32_t a, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(a), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Bounded wait for the phase with the given parity to complete.
-// try_wait suspends the warp in hardware (up to the hint) instead of
-// spinning, so waiting warps leave the issue slots to the other roles.
-__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(a), "r"(parity), "r"(1000u)
-        : "memory");
-    return ok != 0;
-}
-__device__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t *ctrl, uint32_t item) {
-    for (uint32_t it = 0; it < kSpinLimit; ++it) {
-        if (mbar_try(a, parity)) return true;
-        if ((it & 15u) == 15u && ld_relaxed(ctrl + kCtrlError) != 0u) return false;
-    }
-    report_timeout(ctrl, item);
-    return false;
-}
-
-__device__ __forceinline__ unsigned long long ld_relaxed64(const unsigned long long *p) {
-    unsigned long long v;
-    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-    return v;
-}
 
 // ================================================================ mix role
 __device__ void mix_role(const PipeParams &P, unsigned char *sm) {
-    set_role_regs<kMixRegs>();
+    set_role_regs<kMixRegs, kLaunchRegs>();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = lane / kGS, lig = lane % kGS;
     const uint32_t lx = (uint32_t)lig << 4;
@@ -583,7 +519,7 @@ __device__ void copy_tile(const PipeParams &P, unsigned char *sm, int b, const T
 }
 
 __device__ void stage_role(const PipeParams &P, unsigned char *sm, uint32_t ready) {
-    set_role_regs<kStageRegs>();
+    set_role_regs<kStageRegs, kLaunchRegs>();
     const int st = threadIdx.x - kMixT;
     const uint32_t bars = smem_u32(sm + P.off_bar);
     uint4 pre[2 * kStageU];
@@ -749,7 +685,7 @@ __device__ __forceinline__ void unit_flush(const PipeParams &P, uint32_t u, floa
 }
 
 __device__ void pool_role(const PipeParams &P, uint32_t ready, uint32_t drop) {
-    set_role_regs<kPoolRegs>();
+    set_role_regs<kPoolRegs, kLaunchRegs>();
     const int pw = (threadIdx.x - kMixT - kStageT) >> 5, lane = threadIdx.x & 31;
     const int blk = pw * P.cpw + (lane & (P.cpw - 1)), r = lane / P.cpw;
     const bool own = blk < (P.C >> 3);
