@@ -57,6 +57,29 @@ typedef enum moce_status {
 typedef enum moce_dtype { MOCE_F32 = 0, MOCE_BF16 = 1 } moce_dtype_t;
 typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
 
+/*
+ * Kernel path of one layer forward (moce_forward_path). Every path computes
+ * the same layer (Sec. 3.2-3.4) and gives the same results within bf16
+ * output rounding; they differ in how x travels through the GPU.
+ *   MOCE_PATH_AUTO      the fastest path that supports the arguments
+ *   MOCE_PATH_PIPE      one warp-specialised persistent kernel (NHWC bf16,
+ *                       8 <= C_in <= 256, C_in % 8 == 0, k <= 16)
+ *   MOCE_PATH_TWO_PASS  a pooling+gate kernel, then a mixing kernel that
+ *                       stages x through a shared-memory ring (NHWC bf16,
+ *                       as PIPE and C_out <= 64)
+ *   MOCE_PATH_FUSED     the two-group persistent kernel (NHWC bf16,
+ *                       C_in % 8 == 0, k <= 16, shared memory permitting)
+ *   MOCE_PATH_STEPS     one kernel per step: pool, gate, mix (any layout
+ *                       and dtype)
+ */
+typedef enum moce_path {
+    MOCE_PATH_AUTO = 0,
+    MOCE_PATH_PIPE = 1,
+    MOCE_PATH_TWO_PASS = 2,
+    MOCE_PATH_FUSED = 3,
+    MOCE_PATH_STEPS = 4
+} moce_path_t;
+
 /* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */
 typedef struct CUstream_st *moce_stream_t;
 
@@ -158,8 +181,9 @@ moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
  *   aligned, zero-filled before its first use (moce_workspace_init); one
  *   workspace serves one stream at a time.
  * NHWC bf16 with C_in % 8 == 0 and 16-byte aligned x runs one fused
- * persistent kernel; other layouts/dtypes run a sequence of kernels.
- * Asynchronous; device-side failures of the fused kernel (a bounded wait
+ * persistent kernel; other layouts/dtypes run a sequence of kernels (the
+ * choice is moce_forward_path's MOCE_PATH_AUTO).
+ * Asynchronous; device-side failures of the fused kernels (a bounded wait
  * that ran out) are reported by moce_check_device_error.
  */
 moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
@@ -168,6 +192,21 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
                            const float *W1, const float *b1, const float *w2, const float *b2,
                            float tau_min, float tau_max, void *y, void *ws, size_t ws_bytes,
                            moce_stream_t stream);
+
+/*
+ * moce_forward on a chosen kernel path (moce_path_t). Same arguments,
+ * ownership and results as moce_forward; `path` outside the enum is
+ * MOCE_ERR_INVALID_VALUE, and a path that cannot run these arguments
+ * (dtype, layout, C_in, C_out, k, alignment of x) is MOCE_ERR_UNSUPPORTED,
+ * returned before anything is enqueued. For comparing and testing the paths.
+ */
+moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                moce_dtype_t dtype, moce_layout_t layout,
+                                const int32_t *packed_idx, const float *packed_logits,
+                                const int32_t *resid_idx, int n_resid, const float *W1,
+                                const float *b1, const float *w2, const float *b2, float tau_min,
+                                float tau_max, void *y, void *ws, size_t ws_bytes,
+                                moce_path_t path, moce_stream_t stream);
 
 /*
  * The layer forward for callers that cannot allocate device memory: code
@@ -211,6 +250,17 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
  */
 const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                 moce_dtype_t dtype, moce_layout_t layout);
+
+/*
+ * moce_forward_launches and moce_forward_kernel for moce_forward_path with
+ * `path`: 0 / NULL where that path cannot run the arguments. The two-pass
+ * path is named "moce_poolgate_kernel+moce_ring_kernel" (2 launches).
+ */
+int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                               moce_dtype_t dtype, moce_layout_t layout, moce_path_t path);
+const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_in, int C_out,
+                                     int k, moce_dtype_t dtype, moce_layout_t layout,
+                                     moce_path_t path);
 
 /*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word the

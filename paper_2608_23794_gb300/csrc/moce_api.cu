@@ -128,14 +128,36 @@ moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
                                    reinterpret_cast<cudaStream_t>(stream)));
 }
 
-moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
-                           moce_dtype_t dtype, moce_layout_t layout, const int32_t *packed_idx,
-                           const float *packed_logits, const int32_t *resid_idx, int n_resid,
-                           const float *W1, const float *b1, const float *w2, const float *b2,
-                           float tau_min, float tau_max, void *y, void *ws, size_t ws_bytes,
-                           moce_stream_t stream) {
+// Which kernel path serves these arguments when the caller asks for `want`
+// (MOCE_PATH_AUTO picks the fastest that supports them); MOCE_PATH_AUTO is
+// returned when the requested path cannot run them.
+static moce_path_t pick_path(const void *x, int N, int HW, int C_in, int C_out, int k,
+                             moce_dtype_t dtype, moce_layout_t layout, moce_path_t want) {
+    const bool vec = dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
+                     (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+    const bool pipe = vec && pipe_supported(N, HW, C_in, C_out, k);
+    const bool two = vec && ring_supported(N, HW, C_in, C_out, k);
+    const bool fused = vec && fused_supported(N, HW, C_in, C_out, k);
+    switch (want) {
+        case MOCE_PATH_AUTO:
+            return pipe ? MOCE_PATH_PIPE : fused ? MOCE_PATH_FUSED : MOCE_PATH_STEPS;
+        case MOCE_PATH_PIPE: return pipe ? want : MOCE_PATH_AUTO;
+        case MOCE_PATH_TWO_PASS: return two ? want : MOCE_PATH_AUTO;
+        case MOCE_PATH_FUSED: return fused ? want : MOCE_PATH_AUTO;
+        case MOCE_PATH_STEPS: return want;
+    }
+    return MOCE_PATH_AUTO;
+}
+
+moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                moce_dtype_t dtype, moce_layout_t layout,
+                                const int32_t *packed_idx, const float *packed_logits,
+                                const int32_t *resid_idx, int n_resid, const float *W1,
+                                const float *b1, const float *w2, const float *b2, float tau_min,
+                                float tau_max, void *y, void *ws, size_t ws_bytes,
+                                moce_path_t path, moce_stream_t stream) {
     if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
-        !tau_ok(tau_min, tau_max))
+        !tau_ok(tau_min, tau_max) || path < MOCE_PATH_AUTO || path > MOCE_PATH_STEPS)
         return MOCE_ERR_INVALID_VALUE;
     if (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
     const int HW = H * W;
@@ -146,31 +168,30 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
     if (ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
         return MOCE_ERR_INVALID_VALUE;
     if (gate_smem_bytes(k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    const moce_path_t run = pick_path(x, N, HW, C_in, C_out, k, dtype, layout, path);
+    if (run == MOCE_PATH_AUTO) return MOCE_ERR_UNSUPPORTED;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     unsigned char *wsb = static_cast<unsigned char *>(ws);
+    const uint16_t *xv = static_cast<const uint16_t *>(x);
+    uint16_t *yv = static_cast<uint16_t *>(y);
+    switch (run) {
+        case MOCE_PATH_PIPE:
+            return cuda_status(launch_pipe(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
+                                           resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
+                                           yv, L, wsb, s));
+        case MOCE_PATH_TWO_PASS:
+            return cuda_status(launch_ring(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
+                                           resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
+                                           yv, L, wsb, s));
+        case MOCE_PATH_FUSED:
+            return cuda_status(launch_fused(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
+                                            resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
+                                            yv, L, wsb, s));
+        default: break;
+    }
     float *z = reinterpret_cast<float *>(wsb + L.z);
     float *tau = reinterpret_cast<float *>(wsb + L.tau);
     float *a = reinterpret_cast<float *>(wsb + L.a);
-    const bool vec = dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
-                     (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
-    if (vec && pipe_supported(N, HW, C_in, C_out, k)) {
-        return cuda_status(launch_pipe(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
-                                       packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
-                                       b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
-                                       s));
-    }
-    if (vec && ring_supported(N, HW, C_in, C_out, k)) {
-        return cuda_status(launch_ring(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
-                                       packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
-                                       b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
-                                       s));
-    }
-    if (vec && fused_supported(N, HW, C_in, C_out, k)) {
-        return cuda_status(launch_fused(static_cast<const uint16_t *>(x), N, HW, C_in, C_out, k,
-                                        packed_idx, packed_logits, resid_idx, n_resid, W1, b1, w2,
-                                        b2, tau_min, tau_max, static_cast<uint16_t *>(y), L, wsb,
-                                        s));
-    }
     cudaError_t err = launch_pool(x, N, HW, C_in, dtype, layout, z, L, wsb, s);
     if (err == cudaSuccess)
         err = launch_gate(z, N, C_in, C_out, k, packed_idx, packed_logits, W1, b1, w2, b2, tau_min,
@@ -181,26 +202,55 @@ moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_o
     return cuda_status(err);
 }
 
+moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                           moce_dtype_t dtype, moce_layout_t layout, const int32_t *packed_idx,
+                           const float *packed_logits, const int32_t *resid_idx, int n_resid,
+                           const float *W1, const float *b1, const float *w2, const float *b2,
+                           float tau_min, float tau_max, void *y, void *ws, size_t ws_bytes,
+                           moce_stream_t stream) {
+    return moce_forward_path(x, N, H, W, C_in, C_out, k, dtype, layout, packed_idx, packed_logits,
+                             resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max, y, ws, ws_bytes,
+                             MOCE_PATH_AUTO, stream);
+}
+
 int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                           moce_dtype_t dtype, moce_layout_t layout) {
-    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout)) return 0;
+    return moce_forward_path_launches(x, N, H, W, C_in, C_out, k, dtype, layout, MOCE_PATH_AUTO);
+}
+
+int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                               moce_dtype_t dtype, moce_layout_t layout, moce_path_t path) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
+        path < MOCE_PATH_AUTO || path > MOCE_PATH_STEPS)
+        return 0;
     if (N == 0 || H * W == 0) return 0;
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
-    if (dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
-        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
-        (ring_supported(N, H * W, C_in, C_out, k) || pipe_supported(N, H * W, C_in, C_out, k) ||
-         fused_supported(N, H * W, C_in, C_out, k)))
-        return 1;
-    return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
+    switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
+        case MOCE_PATH_PIPE:
+        case MOCE_PATH_FUSED: return 1;
+        case MOCE_PATH_TWO_PASS: return 2;  // pool+gate, then mix
+        case MOCE_PATH_STEPS: return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
+        default: return 0;
+    }
 }
 
 const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                 moce_dtype_t dtype, moce_layout_t layout) {
-    const int launches = moce_forward_launches(x, N, H, W, C_in, C_out, k, dtype, layout);
-    if (launches == 0) return nullptr;
-    if (launches > 1) return "pool+gate+mix";
-    if (pipe_supported(N, H * W, C_in, C_out, k)) return "moce_pipe_kernel";
-    return ring_supported(N, H * W, C_in, C_out, k) ? "moce_ring_kernel" : "moce_fused_kernel";
+    return moce_forward_path_kernel(x, N, H, W, C_in, C_out, k, dtype, layout, MOCE_PATH_AUTO);
+}
+
+const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_in, int C_out,
+                                     int k, moce_dtype_t dtype, moce_layout_t layout,
+                                     moce_path_t path) {
+    if (moce_forward_path_launches(x, N, H, W, C_in, C_out, k, dtype, layout, path) == 0)
+        return nullptr;
+    switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
+        case MOCE_PATH_PIPE: return "moce_pipe_kernel";
+        case MOCE_PATH_TWO_PASS: return "moce_poolgate_kernel+moce_ring_kernel";
+        case MOCE_PATH_FUSED: return "moce_fused_kernel";
+        case MOCE_PATH_STEPS: return "pool+gate+mix";
+        default: return nullptr;
+    }
 }
 
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {

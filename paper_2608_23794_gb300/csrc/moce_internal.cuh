@@ -46,22 +46,22 @@ __host__ __device__ __forceinline__ int pslot(int el, int kp, int i2) {
 }
 __host__ __device__ inline int pslot_count(int R, int kp) { return (R - 1) * (kp >> 1) + ((R - 1) >> 4) + (kp >> 1); }
 
-// Positions per tile of the resident-tile kernel (moce_ring.cu).
+// Positions per tile of the two-pass path (moce_ring.cu).
 constexpr int kRingTile = 64;
 
 struct WsLayout {
     size_t ctrl = 0;      // kCtrlWords uint32
     size_t partial = 0;   // [N][pool_tiles][C] pooling tile sums: fp32 (multi-kernel path) or
                           // tagged 64-bit words {fp32 bits, epoch + 1} (persistent kernels);
-                          // [N][ceil(HW/64)][C] fp32 tile sums for the resident-tile kernel
+                          // [N][ceil(HW/64)][C] tagged fp32 tile sums beyond the fixed-point
+                          // range (two-pass path)
     size_t z = 0;         // [N][C] fp32
     size_t tau = 0;       // [N][R] fp32
     size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit;
-                          // [N][pslot_count][2] fp32 for the resident-tile kernel
-    size_t zacc = 0;      // [2][N][C] int64 fixed-point channel sums (resident-tile kernel;
-                          // two sets, by the parity of the forward's epoch)
-    size_t sync = 0;      // [2][N] tile arrivals, then [2][N] overflow marks, uint32
-                          // (resident-tile kernel)
+                          // softmax weight pairs in mixing-table order (two-pass path)
+    size_t zacc = 0;      // [N][4][C] int64 fixed-point channel sums (two-pass path)
+    size_t sync = 0;      // [2][N] uint32: tile arrivals, then the tag (epoch + 1) of the
+                          // forward that produced example n's weights (two-pass path)
     size_t total = 0;
     int pool_px = 0;
     int pool_tiles = 0;
@@ -79,12 +79,14 @@ inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     auto mx = [](size_t a, size_t b) { return a > b ? a : b; };
     L.ctrl = take(kCtrlWords * 4);
-    L.partial = take((size_t)N * mx((size_t)L.pool_tiles * C * 8, ring_tiles * C * 4));
+    L.partial = take((size_t)N * mx((size_t)L.pool_tiles * C * 8, ring_tiles * C * 8));
     L.z = take((size_t)N * C * 4);
     L.tau = take((size_t)N * R * 4);
-    L.a = take((size_t)N * mx((size_t)R * k * 8, (size_t)pslot_count(R, kp) * 8));
-    L.zacc = take((size_t)2 * N * C * 8);
-    L.sync = take((size_t)N * 16);
+    // two-pass path: a 4 KB weight block per example ([32 pairs][8] float4)
+    (void)kp;
+    L.a = take((size_t)N * mx((size_t)R * k * 8, (size_t)4096));
+    L.zacc = take((size_t)N * 4 * C * 8);
+    L.sync = take((size_t)N * 8);
     L.total = off;
     return L;
 }

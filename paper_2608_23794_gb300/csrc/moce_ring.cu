@@ -1,49 +1,38 @@
-// Resident-tile persistent forward kernel of a MoCE layer (Sec. 3.3-3.4):
-// pooling, gate, softmax weights, routed mixing and the residual expert in
-// one launch that reads x from HBM once, for NHWC bf16 layers with
-// C_in <= 256.
+// Two-pass forward of a MoCE layer (Sec. 3.3-3.4) for NHWC bf16 layers with
+// C_in <= 256, C_out <= 64 and k <= 16.
 //
 // Every expert's temperature depends on the whole-image average of its
 // support (Sec. 3.3), so no position of an example can be mixed before all
-// of the example has been pooled. The example is cut into tiles of 64
-// positions: tile t of example n is work item n*T + t, and CTA b (one per SM,
-// all resident: cooperative launch) takes items b, b + G, b + 2G, ... A tile
-// stays in the CTA's shared memory, transposed to channel-major rows, from
-// the moment it is read until it has been mixed: a ring of D slots holds the
-// CTA's next tiles while the examples they belong to are being pooled by
-// the other CTAs. Four warp roles:
+// of the example has been pooled. The examples are cut into tiles of 64
+// positions (tile t of example n is item n*T + t).
 //
-//   load     (warps 12-27) reads tiles with 16-byte loads (two tiles ahead),
-//            stores each transposed into a free slot and leaves its partial
-//            channel sums in shared memory. It touches no other global
-//            memory, so nothing it does waits for its loads in flight.
-//   publish  (warp 8) adds the partial sums, publishes the tile's channel
-//            sums (fp32 for the exact fallback, and as 64-bit fixed-point
-//            integers added into the example's accumulator) and counts the
-//            tile into the example's arrival counter.
-//   fetch    (warp 9) waits until every tile of its item's example is
-//            counted and reads z from the accumulator (integer sums do not
-//            depend on the order of the additions: z is deterministic) into
-//            one of two z buffers, one item ahead of the gate.
-//   gate     (warps 10-11) evaluates the gate of every expert (Eq. (tau))
-//            and the softmax weights (Eq. (weights)) straight into one of
-//            two mixing tables.
-//   mix      (warps 0-7) mixes a slot with its table: each group of 8 lanes
-//            owns 8 positions per lane and an expert pair (Eq. (expert)) plus
-//            a slice of the residual sum (Eq. (res)); it writes the tile of y
-//            into one of two output buffers and sends it to HBM with one bulk
-//            copy.
+// Pass 1, moce_poolgate_kernel, streams x once at full bandwidth: each CTA
+// reduces a tile to its channel sums and adds them, as 64-bit fixed-point
+// integers, into accumulator words of the example (integer sums do not
+// depend on the order of the additions, so z is deterministic; a sum beyond
+// the fixed-point range is kept as an epoch-tagged fp32 word instead). The
+// CTA that counts an example's last tile reads z, evaluates the gate of
+// every expert (Eq. (tau)) and the softmax weights (Eq. (weights)) and
+// writes them in mixing-table order; it also clears the example's
+// accumulators for the next forward.
 //
-// The roles hand slots, sums and tables over through shared-memory
-// mbarriers; in each role one thread waits and the others block at a
-// barrier. Every wait is bounded: one that gives up records MOCE_ERR_TIMEOUT
-// in the workspace and every other wait returns. The only wait between CTAs
-// is the fetch role's wait for an arrival count; the publish role that
-// counts waits only for its own CTA's loads, so the waits form no cycle.
+// Mixing table: for expert pair p (experts 2p, 2p + 1) and support positions
+// (2 i2, 2 i2 + 1), one float4 {w(2p, 2i2), w(2p, 2i2+1), w(2p+1, 2i2),
+// w(2p+1, 2i2+1)} at entry [p][i2 ^ ((p >> 3) & 3)] of a [32][8] block: the
+// four lane groups of a mixing warp (pairs 8 apart) read different banks.
 //
-// The accumulators and counters of a forward are zeroed by the forward
-// before it (two sets, chosen by the parity of the forward's epoch), so no
-// CTA has to wait for the others to finish reading them.
+// Pass 2, moce_ring_kernel, reads x again and mixes it: one CTA per SM takes
+// items b, b + G, ...; its load warps (8-23) stage each tile, transposed to
+// channel-major rows, into a ring of D shared-memory slots two tiles ahead;
+// the table warps (24-27) copy the item's weights into one of three mixing
+// tables and sum the tile's unselected channels for the residual expert
+// (Eq. (res)); the mix warps (0-7) mix a slot with its table: each group of 8
+// lanes owns 8 positions per lane and one expert pair for the whole launch,
+// whose row offsets it keeps in registers (Eq. (expert)); the tile of y,
+// residual column included, leaves by one bulk copy. The
+// roles hand slots and tables over through shared-memory mbarriers (one
+// thread waits, the others block at a barrier); every wait is bounded and
+// none crosses CTAs.
 #include <algorithm>
 
 #include "moce_device.cuh"
@@ -53,44 +42,80 @@ namespace {
 
 constexpr int kTP = kRingTile;        // positions per tile
 constexpr int kGS = 8;                // lanes of a mixing group
-constexpr int kGPW = 32 / kGS;        // mixing groups per warp
 constexpr int kRB = 16 * kGS;         // bytes per staged channel row (kTP bf16)
 constexpr int kFM = 7;                // chunk swizzle mask of the staged rows
-constexpr int kMixT = 256;            // mix role: warps 0-7
-constexpr int kPubT = 32;             // publish role: warp 8
-constexpr int kFetchT = 32;           // fetch role: warp 9
-constexpr int kGateT = 64;            // gate role: warps 10-11
-constexpr int kLoadT = 512;           // load role: warps 12-27
-constexpr int kRingT = kMixT + kPubT + kFetchT + kGateT + kLoadT;
-constexpr int kGate0 = kMixT + kPubT + kFetchT;  // first gate thread
-constexpr int kLoad0 = kGate0 + kGateT;          // first load thread
+constexpr int kMixT = 256;            // pass 2: mix warps 0-7
+constexpr int kLoadT = 512;           // pass 2: load warps 8-23
+constexpr int kTabT = 128;            // pass 2: table warps 24-27
+constexpr int kRingT = kMixT + kLoadT + kTabT;
+constexpr int kLoad0 = kMixT;                    // first load thread
+constexpr int kTab0 = kMixT + kLoadT;            // first table thread
+constexpr int kResParts = kTabT / 8;             // residual: U entries split kResParts ways
 constexpr int kMixWarps = kMixT / 32;
-constexpr int kGroups = kMixT / kGS;  // mixing groups per CTA
-constexpr int kRPS = kTP + 8;         // row stride (floats) of the residual partial sums
-constexpr int kNT = 2;                // mixing tables
+constexpr int kNT = 3;                // mixing tables
 constexpr int kYB = 2;                // output tile buffers
-constexpr int kNB = 2;                // partial-sum blocks between load and publish
+constexpr int kRS = 4;                // residual columns (the table role runs ahead)
 constexpr int kMaxD = 6;              // x slots at most
-constexpr int kRedF = 1024;           // floats of a partial-sum block
-constexpr int kGateMaxK = 64;
-constexpr int kBarMix = 1, kBarGate = 2, kBarLoad = 3;
-// Fixed-point scale of the pooled sums: 2^24. A tile sum of magnitude at
-// most 2^38 / T keeps the example's integer sum within int64; a larger one
-// marks the example for the exact fp32 reduction instead.
-constexpr float kFixScale = 16777216.0f;
-constexpr float kFixInv = 1.0f / 16777216.0f;
-static_assert(kRingT * 72 <= 65536, "72 registers per thread at one CTA per SM");
+constexpr int kGateMaxK = 16;          // support positions a mixing lane keeps in registers
+constexpr int kMaxPairs = 32;          // expert pairs: one per mixing group
+constexpr int kWBlock = kMaxPairs * 8; // float4 entries of a weight block
+constexpr int kBarMix = 1, kBarLoad = 2, kBarTab = 3;
+// Registers per thread: the launch gives every thread 72 (kRingT * 72 <=
+// 65536); the roles then trade them with setmaxnreg within that total (the
+// mixing loop keeps its row offsets in registers).
+constexpr int kLaunchRegs = 72, kMixRegs = 96, kLoadRegs = 64, kTabRegs = 56;
+static_assert(kMixT * kMixRegs + kLoadT * kLoadRegs + kTabT * kTabRegs <= kRingT * kLaunchRegs,
+              "register split exceeds the launch allocation");
+static_assert(kMixT % 128 == 0 && kLoadT % 128 == 0 && kTabT % 128 == 0, "whole warpgroups");
+constexpr int kPoolT = 256;           // pass 1 threads per CTA
+constexpr int kPoolCTAs = 8;          // pass 1 CTAs per SM
+constexpr int kAccG = 4;              // accumulator words per (example, channel)
+static_assert(kRingT * kLaunchRegs <= 65536, "launch registers at one CTA per SM");
 static_assert(kMixT == 4 * kTP, "four mixing threads per position in the epilogue");
 static_assert(kTP == 8 * kGS, "a group's lanes cover the tile");
+static_assert(kPoolT == 4 * kTP, "pass 1: 32 channel blocks x 8 rows of positions");
 
-// mbarriers (8 bytes each, one arrival each): full[s] (load -> mix),
-// empty[s] (mix -> load), pooled[b] (load -> publish), rfree[b] (publish ->
-// load), tready[b] (gate -> mix), tfree[b] (mix -> gate), zready[b] (fetch
-// -> gate), zfree[b] (gate -> fetch).
-constexpr int kMbFull = 0, kMbEmpty = kMaxD, kMbPooled = 2 * kMaxD, kMbRFree = 2 * kMaxD + kNB,
-              kMbTReady = 2 * kMaxD + 2 * kNB, kMbTFree = 2 * kMaxD + 2 * kNB + kNT,
-              kMbZReady = 2 * kMaxD + 2 * kNB + 2 * kNT,
-              kMbZFree = 2 * kMaxD + 2 * kNB + 3 * kNT, kMbWords = 2 * kMaxD + 2 * kNB + 4 * kNT;
+// Accumulator word of one (example, channel, group): bits 48-55 count the
+// runs published as fp32 instead, bits 0-47 hold the sum of
+// kFixBias + round(s * 2^20) over the fixed-point runs (s = the run's
+// channel sum, |s| < 2^19, so every term is in (0, 2^40) and any count of
+// runs below 256 fits).
+constexpr float kFixScale = 1048576.0f;  // 2^20
+constexpr float kFixInv = 1.0f / 1048576.0f;
+constexpr float kFixMax = 524288.0f;     // 2^19
+constexpr unsigned long long kFixBias = 1ull << 39;
+constexpr unsigned long long kWideOne = 1ull << 48;
+
+// mbarriers of pass 2 (8 bytes each): full[s] (load -> mix, table), empty[s]
+// (mix and table -> load: two arrivals), tready[b] (table -> mix), tfree[b]
+// (mix -> table), rdone[c] (table -> mix: residual column c), rfree[c]
+// (mix -> table).
+constexpr int kMbFull = 0, kMbEmpty = kMaxD, kMbTReady = 2 * kMaxD, kMbTFree = 2 * kMaxD + kNT,
+              kMbRDone = 2 * kMaxD + 2 * kNT, kMbRFree = 2 * kMaxD + 2 * kNT + kRS,
+              kMbWords = 2 * kMaxD + 2 * kNT + 2 * kRS;
+
+// float4 entry of expert pair p, support positions (2 i2, 2 i2 + 1), in a
+// weight block.
+__device__ __forceinline__ int wslot(int p, int i2) { return p * 8 + (i2 ^ ((p >> 3) & 3)); }
+
+struct PoolParams {
+    const uint16_t *x;
+    int N, HW, C, R, k, T;
+    int RL, RPE;                  // tiles per run, runs per example
+    uint32_t runs;                // N * RPE
+    const int32_t *pidx;
+    const float *plog;
+    const float *W1, *b1, *w2, *b2;
+    float tmin, tmax;
+    uint32_t *ctrl;
+    unsigned long long *part;     // [N][RPE][C] tagged fp32 run sums beyond the fixed-point range
+    unsigned long long *zacc;     // [N][kAccG][C] accumulator words
+    uint32_t *count;              // [N] runs of example n counted in this forward
+    uint32_t *made;               // [N] tag of the forward whose pass 1 wrote example n's weights
+    float4 *wts;                  // [N][kWBlock] softmax weights in mixing-table order
+    float *z, *tau;
+    int kp, Kg;
+};
 
 struct RingParams {
     const uint16_t *x;
@@ -98,44 +123,32 @@ struct RingParams {
     int N, HW, C, R, k, nU, T;
     uint32_t items;               // N * T tiles
     const int32_t *pidx;
-    const float *plog;
     const int32_t *resid;
-    const float *W1, *b1, *w2, *b2;
-    float tmin, tmax;
     uint32_t *ctrl;
-    float *part;                  // [N][T][C] tile channel sums (exact fallback)
-    unsigned long long *zacc;     // [2][N][C] fixed-point channel sums of the examples
-    uint32_t *count;              // [2][N] tiles of example n counted
-    uint32_t *ovf;                // [2][N] a tile sum of example n was beyond the fixed-point range
-    float *z, *tau;
+    const float4 *wts;            // [N][kWBlock] from pass 1
+    const uint32_t *made;         // [N] tags written with them
     int D;                        // x slots
-    int CG, nrow;                 // load role: 64-channel groups (1, 2, 4), partial-sum rows
-    int kp, Es, ks, Kg;           // Kg: padded gate width (16, 32), 0: a warp per expert
-    int RS;                       // entries per support position of a mixing table (tslot)
+    int CG;                       // load role: 64-channel groups (1, 2, 4)
+    int kp, Es;
     int bulk_y;                   // output tiles leave by one bulk copy
-    int gate_tabs;                // support tables of the gate in shared memory, [k][R]
-    float fix_max;                // largest tile sum magnitude for the fixed-point path
     uint32_t off_xs, xs_bytes;
     uint32_t off_tab[kNT], off_ys[kYB];
-    uint32_t off_rp, off_red, off_zs, off_uw, off_W1, off_b1, off_w2, off_pidx, off_plog, off_U,
-        off_bar;
+    uint32_t off_res, off_rred, off_U, off_bar;
+    float inv_nU;                 // 1 / |U| (0 when U is empty)
     float inv_E;
 };
 
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p) {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
 __device__ __forceinline__ void red_add_u64(unsigned long long *p, unsigned long long v) {
     asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
-// Bounded wait until *p == want. False when this or another wait gave up.
-__device__ bool wait_count(const uint32_t *p, uint32_t want, uint32_t *ctrl, uint32_t item) {
+
+// Bounded wait for an mbarrier phase; the waiting thread sleeps between
+// polls, so its warp leaves the issue slots to the warps that work.
+__device__ bool ring_wait(uint32_t a, uint32_t parity, uint32_t *ctrl, uint32_t item) {
     for (uint32_t it = 0; it < kSpinLimit; ++it) {
-        if (ld_acquire(p) == want) return true;
-        if (ld_relaxed(ctrl + kCtrlError) != 0u) return false;
-        __nanosleep(it < 64 ? 32 : 256);
+        if (mbar_try(a, parity)) return true;
+        if ((it & 15u) == 15u && ld_relaxed(ctrl + kCtrlError) != 0u) return false;
+        __nanosleep(64);
     }
     report_timeout(ctrl, item);
     return false;
@@ -145,16 +158,7 @@ __device__ __forceinline__ uint32_t mbar(const RingParams &P, const unsigned cha
     return smem_u32(sm + P.off_bar) + 8u * (uint32_t)word;
 }
 
-// Entry (uint4 units) of support positions (2 i2, 2 i2 + 1) of expert e in a
-// mixing table {row offset, row offset, weight, weight}. Entries are grouped
-// by position: a gate warp writing one position of 32 experts touches
-// consecutive entries, and the block of 16 experts shifts the entries by
-// one, so the four lane groups of a mixing warp (experts 16 apart) read
-// different banks.
-__device__ __host__ __forceinline__ int tslot(int RS, int e, int i2) { return i2 * RS + e + (e >> 4); }
-__host__ inline int tslot_rows(int R) { return R + (R >> 4) + 1; }
-
-// Support table element (e, i): [k][R] in shared memory or [R][k] in global.
+// Support table element (e, i): [R][k] in global memory.
 struct SupTab {
     const int32_t *idx;
     const float *lg;
@@ -162,258 +166,239 @@ struct SupTab {
     __device__ __forceinline__ int at(int e, int i) const { return e * se + i * si; }
 };
 
-// ================================================================ gate role
+// ================================================================ pass 1
 // Gate of every expert of one example (Eq. (tau)): u = z at the expert's
 // support in deployment order, h = ReLU(W1 u + b1), g = w2 . h + b2,
 // tau = tau_min + (tau_max - tau_min) sigma(g); weights a = softmax(L / tau)
-// (Eq. (weights)), written into a mixing table. A thread per expert (k <= K):
-// u in registers, W1 transposed in shared memory ([K][K], zero-padded), the
-// hidden units in blocks of 8.
+// (Eq. (weights)), written into the mixing table. Run by the mix role:
+// K / 4 threads per expert (k <= K), thread q of an expert owns hidden units
+// and support positions 4 q .. 4 q + 3. W1 is transposed in shared memory
+// ([K][K], zero-padded, b2 after w2); the softmax uses powers of two,
+// exp((L_i - L_0) / tau) = 2^((L_i - L_0) log2(e) / tau).
+// Not inlined: its registers do not add to those of the mixing loop.
 template <int K>
-__device__ void gate_threads(const RingParams &P, unsigned char *sm, const float *zs,
-                             const SupTab &S, unsigned char *tab, float *tau_out) {
-    const int gt = threadIdx.x - kGate0;
+__device__ __noinline__ void gate_experts(const PoolParams &P, const float *W1t, const float *b1p,
+                                          const float *w2p, const float *zs, const SupTab &S,
+                                          float4 *wts, float *tau_out) {
+    constexpr int TPE = K / 4;             // threads per expert
+    constexpr int EPP = kPoolT / TPE;      // experts per pass
+    const int st = threadIdx.x;
+    const int q = st % TPE, el = st / TPE;
     const int k = P.k, kp = P.kp;
-    const float *W1t = reinterpret_cast<const float *>(sm + P.off_W1);
-    const float *b1p = reinterpret_cast<const float *>(sm + P.off_b1);
-    const float *w2p = reinterpret_cast<const float *>(sm + P.off_w2);
-    const float b2 = __ldg(P.b2);
-    for (int e = gt; e < P.R; e += kGateT) {
-        float u[K];
+    const float b2 = w2p[K];
+    const float4 bq = *reinterpret_cast<const float4 *>(b1p + 4 * q);
+    const float4 wq = *reinterpret_cast<const float4 *>(w2p + 4 * q);
+    for (int e0 = 0; e0 < P.R; e0 += EPP) {
+        const int e = e0 + el;
+        const bool act = e < P.R;
+        float2 h0 = make_float2(bq.x, bq.y), h1 = make_float2(bq.z, bq.w);
+        // the inputs in blocks of 16
 #pragma unroll
-        for (int i = 0; i < K; ++i) u[i] = i < k ? zs[S.idx[S.at(e, i)]] : 0.f;
-        float g = 0.f;
+        for (int i0 = 0; i0 < K; i0 += 16) {
+            float u[16];
 #pragma unroll
-        for (int jc = 0; jc < K; jc += 8) {
-            float h[8];
+            for (int i = 0; i < 16; ++i)
+                u[i] = (act && i0 + i < k) ? zs[S.idx[S.at(e, i0 + i)]] : 0.f;
 #pragma unroll
-            for (int jj = 0; jj < 8; ++jj) h[jj] = b1p[jc + jj];
-#pragma unroll
-            for (int i = 0; i < K; ++i) {
-                const float4 wa = *reinterpret_cast<const float4 *>(W1t + i * K + jc);
-                const float4 wb = *reinterpret_cast<const float4 *>(W1t + i * K + jc + 4);
-                h[0] = fmaf(wa.x, u[i], h[0]);
-                h[1] = fmaf(wa.y, u[i], h[1]);
-                h[2] = fmaf(wa.z, u[i], h[2]);
-                h[3] = fmaf(wa.w, u[i], h[3]);
-                h[4] = fmaf(wb.x, u[i], h[4]);
-                h[5] = fmaf(wb.y, u[i], h[5]);
-                h[6] = fmaf(wb.z, u[i], h[6]);
-                h[7] = fmaf(wb.w, u[i], h[7]);
+            for (int i = 0; i < 16; ++i) {
+                const float4 w = *reinterpret_cast<const float4 *>(W1t + (i0 + i) * K + 4 * q);
+                const float2 uu = make_float2(u[i], u[i]);
+                h0 = __ffma2_rn(make_float2(w.x, w.y), uu, h0);
+                h1 = __ffma2_rn(make_float2(w.z, w.w), uu, h1);
             }
-#pragma unroll
-            for (int jj = 0; jj < 8; ++jj) g = fmaf(w2p[jc + jj], fmaxf(h[jj], 0.f), g);
         }
+        float g = wq.x * fmaxf(h0.x, 0.f);
+        g = fmaf(wq.y, fmaxf(h0.y, 0.f), g);
+        g = fmaf(wq.z, fmaxf(h1.x, 0.f), g);
+        g = fmaf(wq.w, fmaxf(h1.y, 0.f), g);
+#pragma unroll
+        for (int o = 1; o < TPE; o <<= 1) g += __shfl_xor_sync(0xffffffffu, g, o);
         const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-(g + b2)));
-        const float rt = 1.f / tau;
-        const float L0 = S.lg[S.at(e, 0)];  // position 0 holds the largest logit
-        float ex[K], s = 0.f;
+        const float rt = 1.4426950408889634f / tau;  // log2(e) / tau
+        float ex[4], s = 0.f;
+        if (act) {
+            const float L0 = S.lg[S.at(e, 0)];  // position 0 holds the largest logit
 #pragma unroll
-        for (int i = 0; i < K; ++i) {
-            ex[i] = i < k ? expf((S.lg[S.at(e, i)] - L0) * rt) : 0.f;
-            s += ex[i];
+            for (int m = 0; m < 4; ++m) {
+                const int i = 4 * q + m;
+                ex[m] = i < k ? exp2f((S.lg[S.at(e, i)] - L0) * rt) : 0.f;
+                s += ex[m];
+            }
+        } else {
+#pragma unroll
+            for (int m = 0; m < 4; ++m) ex[m] = 0.f;
         }
-        const float inv = 1.f / s;
-        uint4 *te = reinterpret_cast<uint4 *>(tab);
 #pragma unroll
-        for (int i = 0; i < K; i += 2)  // the odd-k pad gets 0
-            if (i < kp)
-                *reinterpret_cast<float2 *>(reinterpret_cast<float *>(te + tslot(P.RS, e, i >> 1)) + 2) =
-                    make_float2(ex[i] * inv, ex[i + 1] * inv);
-        if (tau_out) tau_out[e] = tau;
+        for (int o = 1; o < TPE; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (act) {
+            const float inv = 1.f / s;
+            // positions 4q .. 4q+3 are entries 2q and 2q+1 (the odd-k pad gets 0)
+            // positions 4q .. 4q+3 are entries 2q and 2q+1 (the odd-k pad gets 0)
+            float *wf = reinterpret_cast<float *>(wts);
+            const int pr = e >> 1, half = 2 * (e & 1);
+            if (4 * q < kp)
+                *reinterpret_cast<float2 *>(wf + 4 * wslot(pr, 2 * q) + half) =
+                    make_float2(ex[0] * inv, ex[1] * inv);
+            if (4 * q + 2 < kp)
+                *reinterpret_cast<float2 *>(wf + 4 * wslot(pr, 2 * q + 1) + half) =
+                    make_float2(ex[2] * inv, ex[3] * inv);
+            if (tau_out && q == 0) tau_out[e] = tau;
+        }
     }
 }
 
-// A warp per expert for 32 < k <= 64, a lane per hidden unit (W1 rows
-// padded to ks in shared memory).
-__device__ void gate_warps(const RingParams &P, unsigned char *sm, const float *zs,
-                           const SupTab &S, unsigned char *tab, float *tau_out) {
-    const int gt = threadIdx.x - kGate0;
-    const int warp = gt >> 5, lane = threadIdx.x & 31;
-    float *uw = reinterpret_cast<float *>(sm + P.off_uw) + warp * P.k;
-    const float *W1s = reinterpret_cast<const float *>(sm + P.off_W1);
-    const float *b1s = reinterpret_cast<const float *>(sm + P.off_b1);
-    const float *w2s = reinterpret_cast<const float *>(sm + P.off_w2);
-    const int k = P.k, ks = P.ks, kp = P.kp;
-    const float b2 = __ldg(P.b2);
-    for (int e = warp; e < P.R; e += kGateT / 32) {
-        for (int i = lane; i < k; i += 32) uw[i] = zs[S.idx[S.at(e, i)]];
-        __syncwarp();
-        float gp = 0.f;
-        for (int jj = lane; jj < k; jj += 32) {
-            const float *wr = W1s + jj * ks;
-            float hj = b1s[jj];
-            for (int i = 0; i < k; ++i) hj = fmaf(wr[i], uw[i], hj);
-            gp = fmaf(w2s[jj], fmaxf(hj, 0.f), gp);
+
+// Shared memory of pass 1: partial sums [8][C], z [C], W1 transposed [Kg][Kg],
+// b1 [Kg], w2 [Kg] + b2, the last-CTA flag.
+struct PoolSmem {
+    float red[8 * 256];
+    float zs[256];
+    float W1t[32 * 32];
+    float b1[32];
+    float w2[33];
+    uint32_t last;
+};
+
+// The example's gate, by its last pooling CTA: z from the accumulator words
+// (and the tagged fp32 run sums, in run order), then every expert's
+// temperature and weights; the accumulators and the counter are cleared for
+// the next forward.
+__device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t tag) {
+    const int tid = threadIdx.x;
+    const unsigned long long T = (unsigned long long)P.RPE;  // runs of the example
+    unsigned long long *za = P.zacc + (size_t)n * kAccG * P.C;
+    for (int c = tid; c < P.C; c += kPoolT) {
+        long long fx = 0;
+        bool wide = false;
+#pragma unroll
+        for (int g = 0; g < kAccG; ++g) {
+            const unsigned long long Tg = (T - (unsigned long long)g + kAccG - 1) / kAccG;
+            const unsigned long long w = __ldcg(za + (size_t)g * P.C + c);
+            const unsigned long long wg = (w >> 48) & 0xffull;
+            fx += (long long)(w & ((1ull << 48) - 1ull)) - (long long)((Tg - wg) * kFixBias);
+            wide = wide || wg != 0ull;
         }
-        const float gv = warp_sum(gp) + b2;
-        const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-gv));
-        const float L0 = S.lg[S.at(e, 0)];
-        const float ex0 = lane < k ? expf((S.lg[S.at(e, lane)] - L0) / tau) : 0.f;
-        const float ex1 = lane + 32 < k ? expf((S.lg[S.at(e, lane + 32)] - L0) / tau) : 0.f;
-        const float zsum = warp_sum(ex0 + ex1);
-        float *tw = reinterpret_cast<float *>(tab);
-        if (lane < kp) tw[4 * tslot(P.RS, e, lane >> 1) + 2 + (lane & 1)] = lane < k ? ex0 / zsum : 0.f;
-        if (lane + 32 < kp)
-            tw[4 * tslot(P.RS, e, (lane + 32) >> 1) + 2 + (lane & 1)] = lane + 32 < k ? ex1 / zsum : 0.f;
-        if (lane == 0 && tau_out) tau_out[e] = tau;
-        __syncwarp();
+        float s = __ll2float_rn(fx) * kFixInv;
+        if (wide) {
+            const unsigned long long *pc = P.part + (size_t)n * P.RPE * P.C + c;
+            for (int t = 0; t < P.RPE; ++t) {
+                const unsigned long long wv = __ldcg(pc + (size_t)t * P.C);
+                if ((uint32_t)(wv >> 32) == tag) s += __uint_as_float((uint32_t)wv);
+            }
+        }
+        const float zv = s / (float)P.HW;
+        S.zs[c] = zv;
+        P.z[(size_t)n * P.C + c] = zv;
+#pragma unroll
+        for (int g = 0; g < kAccG; ++g) za[(size_t)g * P.C + c] = 0ull;
     }
+    // W1 transposed (W1t[i * Kg + j] = W1[j][i]), zero-padded; b2 after w2
+    for (int q = tid; q < P.Kg * P.Kg; q += kPoolT) {
+        const int i = q / P.Kg, j = q - i * P.Kg;
+        S.W1t[q] = (j < P.k && i < P.k) ? __ldg(P.W1 + j * P.k + i) : 0.f;
+    }
+    for (int j = tid; j < P.Kg; j += kPoolT) {
+        S.b1[j] = j < P.k ? __ldg(P.b1 + j) : 0.f;
+        S.w2[j] = j < P.k ? __ldg(P.w2 + j) : 0.f;
+    }
+    if (tid == 0) {
+        S.w2[P.Kg] = __ldg(P.b2);
+        P.count[n] = 0u;
+    }
+    __syncthreads();
+    SupTab sup;
+    sup.idx = P.pidx;
+    sup.lg = P.plog;
+    sup.se = P.k;
+    sup.si = 1;
+    float4 *wts = P.wts + (size_t)n * kWBlock;
+    // entries no expert writes (padding positions, the twin of an odd last
+    // expert) stay 0
+    for (int q = tid; q < kWBlock; q += kPoolT) wts[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+    __syncthreads();
+    float *tau = P.tau + (size_t)n * P.R;
+    if (P.Kg == 16) gate_experts<16>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau);
+    else gate_experts<32>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau);
+    if (tid == 0) P.made[n] = tag;  // read by pass 2 after this kernel ends
 }
 
-// z of item r's example into z buffer r mod 2 (Sec. 3.3, GAP): wait until
-// every tile of the example is counted, then the example's fixed-point
-// accumulator (or, past the fixed-point range, the fp32 tile sums in tile
-// order). Lane l owns channels 8 l .. 8 l + 7. The CTA with the example's
-// first tile also writes z to the workspace.
-__device__ void fetch_role(const RingParams &P, unsigned char *sm, uint32_t par) {
-    const int lane = threadIdx.x & 31;
-    const int c0 = 8 * lane;
-    const bool own = c0 < P.C;
-    const uint32_t *count = P.count + (size_t)par * P.N;
-    const uint32_t *ovf = P.ovf + (size_t)par * P.N;
-    const unsigned long long *zacc = P.zacc + (size_t)par * P.N * P.C;
-    const float inv_hw = 1.0f / (float)P.HW;
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t zb = r & 1u;
-        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
-        bool ok = true;
-        if (lane == 0) {
-            ok = r < 2u || mbar_wait(mbar(P, sm, kMbZFree + zb), ((r >> 1) - 1u) & 1u, P.ctrl, it);
-            ok = ok && wait_count(count + n, (uint32_t)P.T, P.ctrl, it);
-        }
-        if (!__all_sync(0xffffffffu, ok)) break;
-        __syncwarp();
-        float z[8];
-        if (own) {
-            const ulonglong2 *za = reinterpret_cast<const ulonglong2 *>(zacc + (size_t)n * P.C + c0);
-            const ulonglong2 q0 = __ldcg(za), q1 = __ldcg(za + 1), q2 = __ldcg(za + 2),
-                             q3 = __ldcg(za + 3);
-            const unsigned long long q[8] = {q0.x, q0.y, q1.x, q1.y, q2.x, q2.y, q3.x, q3.y};
-#pragma unroll
-            for (int m = 0; m < 8; ++m) z[m] = __ll2float_rn((long long)q[m]) * kFixInv * inv_hw;
-        }
-        if (__ldcg(ovf + n) != 0u && own) {
-            // a tile sum was beyond the fixed-point range: the fp32 tile sums
+// A CTA pools one run of up to RL consecutive tiles of one example: thread
+// (row = tid / 32, cb = tid mod 32) adds positions row, row + 8, ... of
+// channels 8 cb .. 8 cb + 7 over the run (eight 16-byte loads in flight per
+// tile), the eight rows are added in order through shared memory, and thread
+// c publishes channel c of the run. The CTA that counts an example's last
+// run finishes the example.
+__global__ void __launch_bounds__(kPoolT) moce_poolgate_kernel(const PoolParams P) {
+    __shared__ __align__(16) PoolSmem S;
+    const int tid = threadIdx.x;
+    const int row = tid >> 5, cb = tid & 31;
+    const bool own = 8 * cb < P.C;
+    const uint32_t tag = ld_relaxed(P.ctrl + kCtrlEpoch) + 1u;
+    const uint32_t drop = ld_relaxed(P.ctrl + kCtrlDropItem);
+    for (uint32_t ru = blockIdx.x; ru < P.runs; ru += gridDim.x) {
+        const int n = (int)(ru / (uint32_t)P.RPE), j = (int)(ru - (uint32_t)n * P.RPE);
+        const int t0 = j * P.RL, t1 = min(P.T, t0 + P.RL);
+        const uint16_t *xe = P.x + (size_t)n * P.HW * P.C + 8 * cb;
+        float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int t = t0; t < t1; ++t) {
+            const int p0 = t * kTP, np = min(kTP, P.HW - p0);
+            uint4 v[8];
 #pragma unroll
             for (int m = 0; m < 8; ++m) {
-                const float *pc = P.part + (size_t)n * P.T * P.C + c0 + m;
-                float s = 0.f;
-                for (int tt = 0; tt < P.T; ++tt) s += __ldcg(pc + (size_t)tt * P.C);
-                z[m] = s / (float)P.HW;
+                const int p = row + 8 * m;
+                v[m] = (own && p < np) ? ld_stream(xe + (size_t)(p0 + p) * P.C)
+                                       : make_uint4(0u, 0u, 0u, 0u);
             }
-        }
-        if (own) {
-            float4 *zs = reinterpret_cast<float4 *>(reinterpret_cast<float *>(sm + P.off_zs) +
-                                                    zb * P.C + c0);
-            zs[0] = make_float4(z[0], z[1], z[2], z[3]);
-            zs[1] = make_float4(z[4], z[5], z[6], z[7]);
-            if (t == 0) {
-                float4 *zo = reinterpret_cast<float4 *>(P.z + (size_t)n * P.C + c0);
-                zo[0] = zs[0];
-                zo[1] = zs[1];
-            }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(mbar(P, sm, kMbZReady + zb));
-    }
-}
-
-// The gate of item r from z buffer r mod 2 into table r mod kNT. The CTA
-// with the example's first tile also writes tau to the workspace.
-__device__ void gate_role(const RingParams &P, unsigned char *sm) {
-    const int gt = threadIdx.x - kGate0;
-    SupTab S;
-    if (P.gate_tabs) {
-        S.idx = reinterpret_cast<const int32_t *>(sm + P.off_pidx);
-        S.lg = reinterpret_cast<const float *>(sm + P.off_plog);
-        S.se = 1;
-        S.si = P.R;
-    } else {
-        S.idx = P.pidx;
-        S.lg = P.plog;
-        S.se = P.k;
-        S.si = 1;
-    }
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t tb = r % kNT, zb = r & 1u;
-        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
-        bool ok = true;
-        if (gt == 0) {
-            // table tb is free once the mix role is done with item r - kNT
-            ok = r < kNT ||
-                 mbar_wait(mbar(P, sm, kMbTFree + tb), ((r / kNT) - 1u) & 1u, P.ctrl, it);
-            ok = ok && mbar_wait(mbar(P, sm, kMbZReady + zb), (r >> 1) & 1u, P.ctrl, it);
-        }
-        if (!bar_and(kBarGate, kGateT, ok)) break;
-        const float *zs = reinterpret_cast<const float *>(sm + P.off_zs) + zb * P.C;
-        unsigned char *tab = sm + P.off_tab[tb];
-        float *tau_out = t == 0 ? P.tau + (size_t)n * P.R : nullptr;
-        if (P.Kg == 16) gate_threads<16>(P, sm, zs, S, tab, tau_out);
-        else if (P.Kg == 32) gate_threads<32>(P, sm, zs, S, tab, tau_out);
-        else gate_warps(P, sm, zs, S, tab, tau_out);
-        bar_sync(kBarGate, kGateT);  // the table is complete; the z buffer is free again
-        if (gt == 0) {
-            mbar_arrive(mbar(P, sm, kMbTReady + tb));
-            mbar_arrive(mbar(P, sm, kMbZFree + zb));
-        }
-    }
-}
-
-// Publishes the channel sums of item r's tile (partial sums of block r mod
-// kNB) and counts the tile into its example: lane l owns channels 8 l ..
-// 8 l + 7.
-__device__ void publish_role(const RingParams &P, unsigned char *sm, uint32_t par,
-                             uint32_t drop) {
-    const int lane = threadIdx.x & 31;
-    const int c0 = 8 * lane;
-    const bool own = c0 < P.C;
-    uint32_t *count = P.count + (size_t)par * P.N;
-    uint32_t *ovf = P.ovf + (size_t)par * P.N;
-    unsigned long long *zacc = P.zacc + (size_t)par * P.N * P.C;
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t b = r % kNB;
-        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
-        bool ok = true;
-        if (lane == 0) ok = mbar_wait(mbar(P, sm, kMbPooled + b), (r / kNB) & 1u, P.ctrl, it);
-        if (!__all_sync(0xffffffffu, ok)) break;
-        __syncwarp();  // lane 0's wait orders the partial sums before every lane's reads
-        if (own) {
-            const float *red = reinterpret_cast<const float *>(sm + P.off_red) + b * kRedF;
-            float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            for (int q = 0; q < P.nrow; ++q) {
-                const float4 a = *reinterpret_cast<const float4 *>(red + q * P.C + c0);
-                const float4 c = *reinterpret_cast<const float4 *>(red + q * P.C + c0 + 4);
-                v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
-                v[4] += c.x; v[5] += c.y; v[6] += c.z; v[7] += c.w;
-            }
-            float4 *pt = reinterpret_cast<float4 *>(P.part + ((size_t)n * P.T + t) * P.C + c0);
-            pt[0] = make_float4(v[0], v[1], v[2], v[3]);
-            pt[1] = make_float4(v[4], v[5], v[6], v[7]);
-            bool big = false;
 #pragma unroll
             for (int m = 0; m < 8; ++m) {
-                if (fabsf(v[m]) <= P.fix_max)
-                    red_add_u64(zacc + (size_t)n * P.C + c0 + m,
-                                (unsigned long long)__float2ll_rn(v[m] * kFixScale));
-                else
-                    big = true;  // also NaN
+                a[0] += bf16lo(v[m].x); a[1] += bf16hi(v[m].x);
+                a[2] += bf16lo(v[m].y); a[3] += bf16hi(v[m].y);
+                a[4] += bf16lo(v[m].z); a[5] += bf16hi(v[m].z);
+                a[6] += bf16lo(v[m].w); a[7] += bf16hi(v[m].w);
             }
-            if (big) atomicOr(ovf + n, 1u);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(mbar(P, sm, kMbRFree + b));  // block b is read
-        __threadfence();
-        __syncwarp();
-        if (lane == 0 && it + 1u != drop)  // fault injection: this tile is never counted
-            atomicAdd(count + n, 1u);
+        if (own) {
+            float4 *rr = reinterpret_cast<float4 *>(S.red + row * P.C + 8 * cb);
+            rr[0] = make_float4(a[0], a[1], a[2], a[3]);
+            rr[1] = make_float4(a[4], a[5], a[6], a[7]);
+        }
+        __syncthreads();
+        if (tid < P.C && ru + 1u != drop) {  // fault injection: this run is never counted
+            float s = 0.f;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) s += S.red[q * P.C + tid];
+            unsigned long long add;
+            if (fabsf(s) < kFixMax) {
+                add = kFixBias + (unsigned long long)__float2ll_rn(s * kFixScale);
+            } else {  // beyond the fixed-point range (or NaN): a tagged fp32 word
+                P.part[((size_t)n * P.RPE + j) * P.C + tid] =
+                    ((unsigned long long)tag << 32) | __float_as_uint(s);
+                add = kWideOne;
+            }
+            red_add_u64(P.zacc + ((size_t)n * kAccG + (j % kAccG)) * P.C + tid, add);
+            __threadfence();
+        }
+        __syncthreads();  // every channel of the run is added; red is free again
+        if (tid == 0) {
+            uint32_t last = 0u;
+            if (ru + 1u != drop) {
+                const uint32_t old = atomicAdd(P.count + n, 1u);
+                if (old == (uint32_t)P.RPE - 1u) {
+                    __threadfence();
+                    last = 1u;
+                }
+            }
+            S.last = last;
+        }
+        __syncthreads();
+        if (S.last) {
+            finish_example(P, S, n, tag);
+            __syncthreads();
+        }
     }
 }
 
-// ================================================================ load role
+// ================================================================ pass 2
 // Staging unit (q, j, cc) of a tile: positions pa = q + 16 j and pa + 8,
 // channels 8 cc .. 8 cc + 7 (two 16-byte loads), stored as eight words of
 // pixel pairs into rows 8 cc .. 8 cc + 7, word j of chunk q ^ (cc & 7). A
@@ -425,7 +410,6 @@ struct LoadUnits {
     int nu;          // units per tile (0..2)
     int cc;          // 8-channel block
     bool own;        // cc < C / 8
-    int row;         // row of the partial-sum block
     int pa[2];       // low position of each unit (the high one is pa + 8)
     int src[2];      // element offset of the low position's load in a tile of x
     int dst[2];      // byte offset of the unit's first word in a slot
@@ -438,7 +422,6 @@ __device__ __forceinline__ LoadUnits load_units(const RingParams &P, int lt) {
     u.cc = 8 * (w & (P.CG - 1)) + (lane & 7);
     u.own = u.cc < (P.C >> 3);
     u.nu = (w < 8 * P.CG) + (w + 16 < 8 * P.CG);
-    u.row = w / P.CG;
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
         const int q = (w + 16 * i) / P.CG;
@@ -470,66 +453,36 @@ __device__ __forceinline__ void tile_loads(const RingParams &P, const LoadUnits 
     }
 }
 
-// One item of the load role: store the tile held in v into slot r mod D,
-// refill v with the loads of the item two ahead, leave the tile's partial
-// channel sums (one row per warp row) in block r mod kNB. False when a wait
-// gave up.
+// One item of the load role: store the tile held in v into slot r mod D and
+// refill v with the loads of the item two ahead. False when a wait gave up.
 __device__ __forceinline__ bool load_item(const RingParams &P, unsigned char *sm,
                                           const LoadUnits &u, uint32_t it, uint32_t r, uint4 *v) {
     const int lt = threadIdx.x - kLoad0;
-    const int lane = lt & 31;
-    const uint32_t s = r % (uint32_t)P.D, b = r % kNB;
-    // slot s is free once the mix role is done with item r - D, block b once
-    // the publish role is done with item r - kNB
+    const uint32_t s = r % (uint32_t)P.D;
+    // slot s is free once the mix role is done with item r - D
     bool ok = true;
-    if (lt == 0) {
-        if (r >= (uint32_t)P.D)
-            ok = mbar_wait(mbar(P, sm, kMbEmpty + s), ((r / P.D) - 1u) & 1u, P.ctrl, it);
-        if (ok && r >= (uint32_t)kNB)
-            ok = mbar_wait(mbar(P, sm, kMbRFree + b), ((r / kNB) - 1u) & 1u, P.ctrl, it);
-    }
+    if (lt == 0 && r >= (uint32_t)P.D)
+        ok = ring_wait(mbar(P, sm, kMbEmpty + s), ((r / P.D) - 1u) & 1u, P.ctrl, it);
     if (!bar_and(kBarLoad, kLoadT, ok)) return false;
     unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
-    float acc[8];
-#pragma unroll
-    for (int m = 0; m < 8; ++m) acc[m] = 0.f;
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
         if (i >= u.nu || !u.own) continue;
         unsigned char *d = xs + u.dst[i];
         const uint4 va = v[2 * i], vb = v[2 * i + 1];
-        uint32_t w[8];
-        w[0] = __byte_perm(va.x, vb.x, 0x5410); w[1] = __byte_perm(va.x, vb.x, 0x7632);
-        w[2] = __byte_perm(va.y, vb.y, 0x5410); w[3] = __byte_perm(va.y, vb.y, 0x7632);
-        w[4] = __byte_perm(va.z, vb.z, 0x5410); w[5] = __byte_perm(va.z, vb.z, 0x7632);
-        w[6] = __byte_perm(va.w, vb.w, 0x5410); w[7] = __byte_perm(va.w, vb.w, 0x7632);
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-            *reinterpret_cast<uint32_t *>(d + m * kRB) = w[m];
-            acc[m] += bf16lo(w[m]) + bf16hi(w[m]);
-        }
+        *reinterpret_cast<uint32_t *>(d + 0 * kRB) = __byte_perm(va.x, vb.x, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 1 * kRB) = __byte_perm(va.x, vb.x, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 2 * kRB) = __byte_perm(va.y, vb.y, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 3 * kRB) = __byte_perm(va.y, vb.y, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 4 * kRB) = __byte_perm(va.z, vb.z, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 5 * kRB) = __byte_perm(va.z, vb.z, 0x7632);
+        *reinterpret_cast<uint32_t *>(d + 6 * kRB) = __byte_perm(va.w, vb.w, 0x5410);
+        *reinterpret_cast<uint32_t *>(d + 7 * kRB) = __byte_perm(va.w, vb.w, 0x7632);
     }
-    // the item two ahead is in flight while this one is reduced and the
-    // next one is stored
+    // the item two ahead is in flight while the next one is stored
     tile_loads(P, u, it + 2u * gridDim.x, v);
-    // partial channel sums: lanes with the same cc (j = 0..3) by shuffles;
-    // the publish role adds the rows
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-        acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], 8);
-        acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], 16);
-    }
-    if (lane < 8 && u.nu > 0 && u.own) {
-        float *red = reinterpret_cast<float *>(sm + P.off_red) + b * kRedF;
-        float4 *rr = reinterpret_cast<float4 *>(red + u.row * P.C + u.cc * 8);
-        rr[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-        rr[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
-    }
     bar_sync(kBarLoad, kLoadT);
-    if (lt == 0) {
-        mbar_arrive(mbar(P, sm, kMbFull + s));
-        mbar_arrive(mbar(P, sm, kMbPooled + b));
-    }
+    if (lt == 0) mbar_arrive(mbar(P, sm, kMbFull + s));
     return true;
 }
 
@@ -537,6 +490,7 @@ __device__ __forceinline__ bool load_item(const RingParams &P, unsigned char *sm
 // set stays in registers).
 __device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnits &u, uint4 *va,
                           uint4 *vb) {
+    set_role_regs<kLoadRegs, kLaunchRegs>();
     uint32_t r = 0;
     for (uint32_t it = blockIdx.x; it < P.items;) {
         if (!load_item(P, sm, u, it, r, va)) break;
@@ -549,27 +503,99 @@ __device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnit
     }
 }
 
+// The table role, per item r: copies the weights of the item's example
+// (pass 1) into table r mod kNT (an example whose weights pass 1 of this
+// forward did not produce, because a tile was never counted, is reported as
+// MOCE_ERR_TIMEOUT); then, once the tile is staged, the residual expert
+// (Eq. (res)): thread (q = chunk, part) adds U entries part, part +
+// kResParts, ... for the chunk's 8 positions, the parts are added in order,
+// and res[r mod kYB][p] = sum / |U| (0 if U is empty).
+__device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag) {
+    set_role_regs<kTabRegs, kLaunchRegs>();
+    const int tt = threadIdx.x - kTab0;
+    const int q = tt & 7, part = tt >> 3;
+    const uint32_t lx = (uint32_t)q << 4;
+    const int32_t *s_resid = reinterpret_cast<const int32_t *>(sm + P.off_U);
+    float *rred = reinterpret_cast<float *>(sm + P.off_rred);
+    uint32_t r = 0;
+    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
+        const uint32_t tb = r % kNT, s = r % (uint32_t)P.D, rc = r % kRS;
+        const int n = (int)(it / (uint32_t)P.T);
+        bool ok = true;
+        if (tt == 0 && r >= (uint32_t)kNT)
+            ok = ring_wait(mbar(P, sm, kMbTFree + tb), ((r / kNT) - 1u) & 1u, P.ctrl, it);
+        if (!bar_and(kBarTab, kTabT, ok)) break;
+        if (tt == 0 && __ldg(P.made + n) != tag) report_timeout(P.ctrl, it);
+        {
+            const float4 *wn = P.wts + (size_t)n * kWBlock;
+            float4 *tab = reinterpret_cast<float4 *>(sm + P.off_tab[tb]);
+            float4 w[kWBlock / kTabT];
+#pragma unroll
+            for (int j = 0; j < kWBlock / kTabT; ++j) w[j] = __ldg(wn + tt + kTabT * j);
+#pragma unroll
+            for (int j = 0; j < kWBlock / kTabT; ++j) tab[tt + kTabT * j] = w[j];
+        }
+        bar_sync(kBarTab, kTabT);
+        if (tt == 0) {
+            mbar_arrive(mbar(P, sm, kMbTReady + tb));
+            ok = ring_wait(mbar(P, sm, kMbFull + s), (r / P.D) & 1u, P.ctrl, it);
+            if (ok && r >= (uint32_t)kRS)
+                ok = ring_wait(mbar(P, sm, kMbRFree + rc), ((r / kRS) - 1u) & 1u, P.ctrl, it);
+        }
+        if (!bar_and(kBarTab, kTabT, ok)) break;
+        const unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
+        float2 r0 = make_float2(0.f, 0.f), r1 = r0, r2 = r0, r3 = r0;
+        for (int u = part; u < P.nU; u += kResParts) {
+            const uint32_t c = (uint32_t)s_resid[u];
+            const uint4 vv = lds128(xs + (((c * kRB) | (((c >> 3) & kFM) << 4)) ^ lx));
+            r0 = __fadd2_rn(r0, unpack2(vv.x));
+            r1 = __fadd2_rn(r1, unpack2(vv.y));
+            r2 = __fadd2_rn(r2, unpack2(vv.z));
+            r3 = __fadd2_rn(r3, unpack2(vv.w));
+        }
+        // chunk q's positions are q + 8 m
+        float *rg = rred + part * kTP + q;
+        rg[0 * 8] = r0.x; rg[1 * 8] = r0.y; rg[2 * 8] = r1.x; rg[3 * 8] = r1.y;
+        rg[4 * 8] = r2.x; rg[5 * 8] = r2.y; rg[6 * 8] = r3.x; rg[7 * 8] = r3.y;
+        bar_sync(kBarTab, kTabT);
+        if (tt == 0) mbar_arrive(mbar(P, sm, kMbEmpty + s));  // the slot is read
+        if (tt < kTP) {
+            float sum = 0.f;
+#pragma unroll
+            for (int pp = 0; pp < kResParts; ++pp) sum += rred[pp * kTP + tt];
+            reinterpret_cast<float *>(sm + P.off_res)[rc * kTP + tt] = sum * P.inv_nU;
+        }
+        bar_sync(kBarTab, kTabT);  // rred is free again; the residual column is complete
+        if (tt == 0) mbar_arrive(mbar(P, sm, kMbRDone + rc));
+    }
+}
+
 // ================================================================ mix role
-// Weighted sums of two experts for the lane's 8 positions, over their table
-// entries (RS apart); the experts are interleaved for instruction-level
-// parallelism. An entry is {row offset, row offset, weight, weight} of two
-// support positions.
-__device__ __forceinline__ void mix_pairs(const unsigned char *xs, const uint4 *ta, const uint4 *tb,
-                                          int RS, int npairs, uint32_t lx, float2 &a0, float2 &a1,
-                                          float2 &a2, float2 &a3, float2 &b0, float2 &b1,
-                                          float2 &b2, float2 &b3) {
-#pragma unroll 2
-    for (int i2 = 0; i2 < npairs; ++i2) {
-        const uint4 ea = ta[i2 * RS];
-        const uint4 eb = tb[i2 * RS];
-        const uint4 va0 = lds128(xs + (ea.x ^ lx));
-        const uint4 va1 = lds128(xs + (ea.y ^ lx));
-        const uint4 vb0 = lds128(xs + (eb.x ^ lx));
-        const uint4 vb1 = lds128(xs + (eb.y ^ lx));
-        const float2 wa0 = make_float2(__uint_as_float(ea.z), __uint_as_float(ea.z));
-        const float2 wa1 = make_float2(__uint_as_float(ea.w), __uint_as_float(ea.w));
-        const float2 wb0 = make_float2(__uint_as_float(eb.z), __uint_as_float(eb.z));
-        const float2 wb1 = make_float2(__uint_as_float(eb.w), __uint_as_float(eb.w));
+// Row offset (bytes in a slot) of channel c for the lane whose chunk mask is
+// lx: row c, chunk ((c >> 3) & 7) ^ lane; channel C is the zero row.
+__device__ __forceinline__ uint32_t row_off(uint32_t c, uint32_t lx) {
+    return ((c * kRB) | (((c >> 3) & kFM) << 4)) ^ lx;
+}
+
+// Weighted sums of the lane's expert pair for its 8 positions: per entry i2,
+// one float4 of weights and four 16-byte row chunks whose offsets the lane
+// holds in registers (offs[2 i2]: expert a, positions 2 i2 and 2 i2 + 1, low
+// and high half; offs[2 i2 + 1]: expert b).
+__device__ __forceinline__ void mix_pair_regs(const unsigned char *xs, const float4 *wt, int pr,
+                                              int npairs, const uint32_t *offs, float2 &a0,
+                                              float2 &a1, float2 &a2, float2 &a3, float2 &b0,
+                                              float2 &b1, float2 &b2, float2 &b3) {
+#pragma unroll
+    for (int i2 = 0; i2 < kGateMaxK / 2; ++i2) {
+        if (i2 >= npairs) break;
+        const float4 w = wt[wslot(pr, i2)];
+        const uint32_t oa = offs[2 * i2], ob = offs[2 * i2 + 1];
+        const uint4 va0 = lds128(xs + (oa & 0xffffu));
+        const uint4 va1 = lds128(xs + (oa >> 16));
+        const uint4 vb0 = lds128(xs + (ob & 0xffffu));
+        const uint4 vb1 = lds128(xs + (ob >> 16));
+        const float2 wa0 = make_float2(w.x, w.x), wa1 = make_float2(w.y, w.y);
+        const float2 wb0 = make_float2(w.z, w.z), wb1 = make_float2(w.w, w.w);
         a0 = __ffma2_rn(wa0, unpack2(va0.x), a0);
         a1 = __ffma2_rn(wa0, unpack2(va0.y), a1);
         a2 = __ffma2_rn(wa0, unpack2(va0.z), a2);
@@ -590,40 +616,55 @@ __device__ __forceinline__ void mix_pairs(const unsigned char *xs, const uint4 *
 }
 
 __device__ void mix_role(const RingParams &P, unsigned char *sm) {
+    set_role_regs<kMixRegs, kLaunchRegs>();
     const int st = threadIdx.x;
     const int warp = st >> 5, lane = st & 31;
     const int h = lane / kGS, lig = lane % kGS;
     const uint32_t lx = (uint32_t)lig << 4;
-    const int g = warp * kGPW + h;
     const int R = P.R, E = R + 1, kp = P.kp, NP = (R + 1) >> 1, Es = P.Es;
-    const int32_t *s_resid = reinterpret_cast<const int32_t *>(sm + P.off_U);
-    float *rp = reinterpret_cast<float *>(sm + P.off_rp);
+    const float *res = reinterpret_cast<const float *>(sm + P.off_res);
+    // this group's expert pair (warp w's groups take pairs w + 8h) and its
+    // row offsets, fixed for the whole launch; padding positions and the twin
+    // of an odd last expert read the zero row (their weights are 0)
+    const int pr = warp + kMixWarps * h;
+    const int ea = 2 * pr, eb = ea + 1;
+    const bool pair_on = pr < NP;
+    uint32_t offs[kGateMaxK];
+#pragma unroll
+    for (int i = 0; i < kGateMaxK; i += 2) {
+        uint32_t o[4];
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+            const int e = m < 2 ? ea : eb, pos = i + (m & 1);
+            const uint32_t c = (pair_on && e < R && pos < P.k)
+                                   ? (uint32_t)__ldg(P.pidx + (size_t)e * P.k + pos)
+                                   : (uint32_t)P.C;
+            o[m] = row_off(c, lx);
+        }
+        offs[i] = o[0] | (o[1] << 16);
+        offs[i + 1] = o[2] | (o[3] << 16);
+    }
     uint32_t r = 0;
     for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t s = r % (uint32_t)P.D, tb = r % kNT, yb = r % kYB;
+        const uint32_t s = r % (uint32_t)P.D, tb = r % kNT, yb = r % kYB, rc = r % kRS;
+        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
         // one thread waits for the slot and the table, the others at the
         // barrier; thread 0 has also seen the bulk copy of item r - kYB
         // finish reading ys
         bool ok = true;
         if (st == 0) {
-            ok = mbar_wait(mbar(P, sm, kMbFull + s), (r / P.D) & 1u, P.ctrl, it) &&
-                 mbar_wait(mbar(P, sm, kMbTReady + tb), (r / kNT) & 1u, P.ctrl, it);
+            ok = ring_wait(mbar(P, sm, kMbFull + s), (r / P.D) & 1u, P.ctrl, it) &&
+                 ring_wait(mbar(P, sm, kMbTReady + tb), (r / kNT) & 1u, P.ctrl, it) &&
+                 ring_wait(mbar(P, sm, kMbRDone + rc), (r / kRS) & 1u, P.ctrl, it);
         }
         if (!bar_and(kBarMix, kMixT, ok)) break;
         const unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
         uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[yb]);
-        const uint4 *tab = reinterpret_cast<const uint4 *>(sm + P.off_tab[tb]);
-        // expert pairs: warp w's groups take pairs w + 8h of each block of 32
-        for (int blk = 0; blk < NP; blk += kMixWarps * kGPW) {
-            const int pr = blk + warp + kMixWarps * h;
-            if (pr >= NP) continue;
-            const int ea = 2 * pr, eb = ea + 1;
+        const float4 *wt = reinterpret_cast<const float4 *>(sm + P.off_tab[tb]);
+        if (pair_on) {
             float2 a0 = make_float2(0.f, 0.f), a1 = a0, a2 = a0, a3 = a0;
             float2 b0 = a0, b1 = a0, b2 = a0, b3 = a0;
-            // an odd last expert pairs with itself; its twin's result is dropped
-            const int ebb = eb < R ? eb : ea;
-            mix_pairs(xs, tab + tslot(P.RS, ea, 0), tab + tslot(P.RS, ebb, 0), P.RS, kp >> 1, lx,
-                      a0, a1, a2, a3, b0, b1, b2, b3);
+            mix_pair_regs(xs, wt, pr, kp >> 1, offs, a0, a1, a2, a3, b0, b1, b2, b3);
             // lane lig's positions are lig + 8 m
             if (P.bulk_y) {
                 // rows of odd length: 16-bit stores
@@ -636,6 +677,14 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
                     yh[q * stp] = f32_to_bf16(av[q]);
                     if (eb < R) yh[q * stp + 1] = f32_to_bf16(bv[q]);
                 }
+            } else if (eb == R) {
+                // odd R: the twin's column is the residual column, written
+                // below by another thread
+                uint16_t *yh = ys + lig * Es + ea;
+                const int stp = kGS * Es;
+                const float av[8] = {a0.x, a0.y, a1.x, a1.y, a2.x, a2.y, a3.x, a3.y};
+#pragma unroll
+                for (int q = 0; q < 8; ++q) yh[q * stp] = f32_to_bf16(av[q]);
             } else {
                 uint32_t *yw = reinterpret_cast<uint32_t *>(ys + lig * Es + ea);
                 const int stp = (kGS * Es) >> 1;
@@ -649,43 +698,9 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
                 yw[7 * stp] = pack_bf16x2(a3.y, b3.y);
             }
         }
-        // residual: group g sums U entries g, g + kGroups, ... for its positions
-        if (P.nU > 0) {
-            float2 r0 = make_float2(0.f, 0.f), r1 = r0, r2 = r0, r3 = r0;
-            for (int uu = g; uu < P.nU; uu += kGroups) {
-                const uint32_t c = (uint32_t)s_resid[uu];
-                const uint4 vv = lds128(xs + (((c * kRB) | (((c >> 3) & kFM) << 4)) ^ lx));
-                r0 = __fadd2_rn(r0, unpack2(vv.x));
-                r1 = __fadd2_rn(r1, unpack2(vv.y));
-                r2 = __fadd2_rn(r2, unpack2(vv.z));
-                r3 = __fadd2_rn(r3, unpack2(vv.w));
-            }
-            float *rg = rp + g * kRPS + lig;
-            rg[0 * kGS] = r0.x; rg[1 * kGS] = r0.y; rg[2 * kGS] = r1.x; rg[3 * kGS] = r1.y;
-            rg[4 * kGS] = r2.x; rg[5 * kGS] = r2.y; rg[6 * kGS] = r3.x; rg[7 * kGS] = r3.y;
-        }
-        bar_sync(kBarMix, kMixT);
-        // the slot and the table are no longer read
-        if (st == 0) {
-            mbar_arrive(mbar(P, sm, kMbEmpty + s));
-            mbar_arrive(mbar(P, sm, kMbTFree + tb));
-        }
-        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
+        // the residual column (table role)
         const int p0 = t * kTP, np = min(kTP, P.HW - p0);
-        {
-            // the residual column: four threads per position add a quarter of
-            // the groups' partial sums each
-            const int px = st >> 2, part = st & 3;
-            float sum = 0.f;
-            if (P.nU > 0) {
-#pragma unroll
-                for (int gg = part; gg < kGroups; gg += 4) sum += rp[gg * kRPS + px];
-                sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-                sum += __shfl_xor_sync(0xffffffffu, sum, 2);
-                sum = sum / (float)P.nU;
-            }
-            if (part == 0 && px < np) ys[px * Es + R] = f32_to_bf16(sum);
-        }
+        if (st < np) ys[st * Es + R] = f32_to_bf16(res[rc * kTP + st]);
         const int cnt = np * E;
         uint16_t *dst = P.y + ((size_t)n * P.HW + p0) * E;
         if (P.bulk_y) {
@@ -693,6 +708,10 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             bar_sync(kBarMix, kMixT);
             if (st == 0) {
+                // the slot, the table and the residual column are read
+                mbar_arrive(mbar(P, sm, kMbEmpty + s));
+                mbar_arrive(mbar(P, sm, kMbTFree + tb));
+                mbar_arrive(mbar(P, sm, kMbRFree + rc));
                 asm volatile(
                     "cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n\t"
                     "cp.async.bulk.commit_group;\n\t"
@@ -703,6 +722,12 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
             continue;
         }
         bar_sync(kBarMix, kMixT);
+        if (st == 0) {
+            // the slot, the table and the residual column are read
+            mbar_arrive(mbar(P, sm, kMbEmpty + s));
+            mbar_arrive(mbar(P, sm, kMbTFree + tb));
+            mbar_arrive(mbar(P, sm, kMbRFree + rc));
+        }
         // rows of y not 16-byte aligned: 16-byte streaming stores between a
         // 16-bit head and tail
         const int head = min(
@@ -735,14 +760,13 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
     if (st == 0 && P.bulk_y) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
-// ================================================================ the kernel
+// ================================================================ the mix kernel
 __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P) {
     extern __shared__ __align__(128) unsigned char sm[];
-    const uint32_t epoch = ld_relaxed(P.ctrl + kCtrlEpoch);
-    const uint32_t par = epoch & 1u;
-    const uint32_t drop = ld_relaxed(P.ctrl + kCtrlDropItem);
     const int tid = threadIdx.x;
-    const bool loader = tid >= kLoad0;
+    const uint32_t epoch = ld_relaxed(P.ctrl + kCtrlEpoch);
+    const uint32_t tag = epoch + 1u;
+    const bool loader = tid >= kLoad0 && tid < kTab0;
     // the load role's first two tiles are in flight during the set-up
     LoadUnits lu;
     uint4 va[4], vb[4];
@@ -751,96 +775,35 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
         tile_loads(P, lu, blockIdx.x, va);
         tile_loads(P, lu, blockIdx.x + gridDim.x, vb);
     }
-    // the next forward's accumulators and counters (the other parity) start
-    // from zero; nothing in this forward uses them
-    {
-        const uint32_t np = par ^ 1u;
-        const size_t gid = (size_t)blockIdx.x * kRingT + tid, gs = (size_t)gridDim.x * kRingT;
-        unsigned long long *za = P.zacc + (size_t)np * P.N * P.C;
-        for (size_t i = gid; i < (size_t)P.N * P.C; i += gs) za[i] = 0ull;
-        for (size_t i = gid; i < (size_t)P.N; i += gs) {
-            P.count[np * P.N + i] = 0u;
-            P.ovf[np * P.N + i] = 0u;
-        }
-    }
-    // set-up: U list, gate parameters and support tables, the mixing tables'
-    // row offsets (weights 0), the zero row of every slot, mbarriers
+    // set-up: U list, the zero row of every slot, mbarriers
     int32_t *s_resid = reinterpret_cast<int32_t *>(sm + P.off_U);
     for (int i = tid; i < P.nU; i += kRingT) s_resid[i] = __ldg(P.resid + i);
-    float *W1s = reinterpret_cast<float *>(sm + P.off_W1);
-    float *b1s = reinterpret_cast<float *>(sm + P.off_b1);
-    float *w2s = reinterpret_cast<float *>(sm + P.off_w2);
-    if (P.Kg) {
-        // W1 transposed: W1s[i * Kg + j] = W1[j][i], zero-padded
-        for (int q = tid; q < P.Kg * P.Kg; q += kRingT) {
-            const int i = q / P.Kg, j = q - i * P.Kg;
-            W1s[q] = (j < P.k && i < P.k) ? __ldg(P.W1 + j * P.k + i) : 0.f;
-        }
-        for (int j = tid; j < P.Kg; j += kRingT) {
-            b1s[j] = j < P.k ? __ldg(P.b1 + j) : 0.f;
-            w2s[j] = j < P.k ? __ldg(P.w2 + j) : 0.f;
-        }
-    } else {
-        for (int q = tid; q < P.k * P.k; q += kRingT) {
-            const int j = q / P.k, i = q - j * P.k;
-            W1s[j * P.ks + i] = __ldg(P.W1 + q);
-        }
-        for (int j = tid; j < P.k; j += kRingT) {
-            b1s[j] = __ldg(P.b1 + j);
-            w2s[j] = __ldg(P.w2 + j);
-        }
-    }
-    if (P.gate_tabs) {
-        // [k][R]: a gate warp's threads (experts) read consecutive words
-        for (int q = tid; q < P.R * P.k; q += kRingT) {
-            const int e = q / P.k, i = q - e * P.k;
-            reinterpret_cast<int32_t *>(sm + P.off_pidx)[i * P.R + e] = __ldg(P.pidx + q);
-            reinterpret_cast<float *>(sm + P.off_plog)[i * P.R + e] = __ldg(P.plog + q);
-        }
-    }
     for (int q = tid; q < P.D * (kRB / 4); q += kRingT) {
         const int d = q / (kRB / 4), w = q - d * (kRB / 4);
         reinterpret_cast<uint32_t *>(sm + P.off_xs + d * P.xs_bytes + (size_t)P.C * kRB)[w] = 0u;
     }
-    for (int q = tid; q < P.R * P.kp; q += kRingT) {
-        const int el = q / P.kp, i = q - el * P.kp;
-        uint32_t off = (uint32_t)P.C * kRB;  // padding entries read the zero row
-        if (i < P.k) {
-            const uint32_t c = (uint32_t)__ldg(P.pidx + (size_t)el * P.k + i);
-            off = (c * kRB) | (((c >> 3) & kFM) << 4);
-        }
-        for (int b = 0; b < kNT; ++b) {
-            uint32_t *w = reinterpret_cast<uint32_t *>(
-                reinterpret_cast<uint4 *>(sm + P.off_tab[b]) + tslot(P.RS, el, i >> 1));
-            w[i & 1] = off;
-            w[2 + (i & 1)] = 0u;
-        }
-    }
     if (tid == 0) {
         for (int d = 0; d < P.D; ++d) {
             mbar_init(mbar(P, sm, kMbFull + d), 1);
-            mbar_init(mbar(P, sm, kMbEmpty + d), 1);
-        }
-        for (int b = 0; b < kNB; ++b) {
-            mbar_init(mbar(P, sm, kMbPooled + b), 1);
-            mbar_init(mbar(P, sm, kMbRFree + b), 1);
+            mbar_init(mbar(P, sm, kMbEmpty + d), 2);
         }
         for (int b = 0; b < kNT; ++b) {
             mbar_init(mbar(P, sm, kMbTReady + b), 1);
             mbar_init(mbar(P, sm, kMbTFree + b), 1);
-            mbar_init(mbar(P, sm, kMbZReady + b), 1);
-            mbar_init(mbar(P, sm, kMbZFree + b), 1);
+        }
+        for (int b = 0; b < kRS; ++b) {
+            mbar_init(mbar(P, sm, kMbRDone + b), 1);
+            mbar_init(mbar(P, sm, kMbRFree + b), 1);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
     if (tid < kMixT) mix_role(P, sm);
-    else if (tid < kMixT + kPubT) publish_role(P, sm, par, drop);
-    else if (tid < kGate0) fetch_role(P, sm, par);
-    else if (!loader) gate_role(P, sm);
-    else load_role(P, sm, lu, va, vb);
+    else if (loader) load_role(P, sm, lu, va, vb);
+    else table_role(P, sm, tag);
 
+    // the last CTA advances the epoch (the tag of the next forward)
     __syncthreads();
     if (tid == 0) {
         __threadfence();
@@ -855,11 +818,9 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
 
 // ---------------------------------------------------------------- host side
 struct RingPlan {
-    int D = 0, CG = 0, nrow = 0, kp = 0, Es = 0, ks = 0, Kg = 0, WE = 0, RS = 0;
+    int D = 0, CG = 0, kp = 0, Es = 0, Kg = 0;
     size_t xs_bytes = 0, off_xs = 0, off_tab[kNT] = {}, off_ys[kYB] = {};
-    size_t off_rp = 0, off_red = 0, off_zs = 0, off_uw = 0, off_W1 = 0, off_b1 = 0;
-    size_t off_w2 = 0, off_pidx = 0, off_plog = 0, off_U = 0, off_bar = 0, smem = 0;
-    bool gate_tabs = false;
+    size_t off_res = 0, off_rred = 0, off_U = 0, off_bar = 0, smem = 0;
 };
 
 int sm_count() {
@@ -869,26 +830,18 @@ int sm_count() {
     return sms;
 }
 
-// Shared memory: D slots of C + 1 staged rows (row C = zeros), kNT mixing
-// tables, kYB output tiles, the residual partial sums, the pooling reduction
-// block, z, the gate's parameters and scratch, U, the mailbox, mbarriers. D
-// is the largest count (at most kMaxD) that fits.
-bool ring_plan(int N, int HW, int C, int R, int k, int G, bool bulk_y, RingPlan *plan) {
-    (void)N;
-    if (C % 8 != 0 || C < 8 || C > 256 || k < 1 || k > kGateMaxK || R < 1 || HW < 1 || G < 1)
+// Shared memory of pass 2: D slots of C + 1 staged rows (row C = zeros), kNT
+// mixing tables, kYB output tiles, the residual partial sums, U, mbarriers.
+// D is the largest count (at most kMaxD) that fits.
+bool ring_plan(int C, int R, int k, bool bulk_y, RingPlan *plan) {
+    if (C % 8 != 0 || C < 8 || C > 256 || k < 1 || k > kGateMaxK || R < 1 || R > 2 * kMaxPairs)
         return false;
-    const int T = (HW + kTP - 1) / kTP;
-    if (T > G) return false;  // an example's tiles on distinct CTAs: at most two rounds apart
     RingPlan p;
     const int cgs = ((C >> 3) + 7) / 8;
     p.CG = cgs <= 1 ? 1 : (cgs <= 2 ? 2 : 4);
-    p.nrow = std::min(8, 16 / p.CG);
     p.kp = k + (k & 1);
     p.Es = bulk_y ? R + 1 : (R + 1) + ((R + 1) & 1);
-    p.ks = (k % 2 == 0) ? k + 1 : k;
-    p.Kg = k <= 16 ? 16 : (k <= 32 ? 32 : 0);
-    p.RS = tslot_rows(R);
-    p.WE = (p.kp >> 1) * p.RS;
+    p.Kg = 16;
     p.xs_bytes = align_up((size_t)(C + 1) * kRB, 128);
     size_t off = 0;
     auto take = [&](size_t bytes, size_t al) {
@@ -897,21 +850,10 @@ bool ring_plan(int N, int HW, int C, int R, int k, int G, bool bulk_y, RingPlan 
         off += bytes;
         return o;
     };
-    for (int b = 0; b < kNT; ++b) p.off_tab[b] = take((size_t)p.WE * 16, 16);
+    for (int b = 0; b < kNT; ++b) p.off_tab[b] = take((size_t)kWBlock * 16, 16);
     for (int b = 0; b < kYB; ++b) p.off_ys[b] = take((size_t)kTP * p.Es * 2, 16);
-    p.off_rp = take((size_t)kGroups * kRPS * 4, 16);
-    p.off_red = take((size_t)kNB * kRedF * 4, 16);
-    p.off_zs = take((size_t)2 * C * 4, 16);
-    p.off_uw = take((size_t)(kGateT / 32) * k * 4, 16);
-    const int kg = p.Kg ? p.Kg : k;
-    p.off_W1 = take((size_t)(p.Kg ? p.Kg * p.Kg : k * p.ks) * 4, 16);
-    p.off_b1 = take((size_t)kg * 4, 16);
-    p.off_w2 = take((size_t)kg * 4, 16);
-    p.gate_tabs = (size_t)R * k * 8 <= 8 * 1024;
-    if (p.gate_tabs) {
-        p.off_pidx = take((size_t)R * k * 4, 16);
-        p.off_plog = take((size_t)R * k * 4, 16);
-    }
+    p.off_res = take((size_t)kRS * kTP * 4, 16);
+    p.off_rred = take((size_t)kResParts * kTP * 4, 16);
     p.off_U = take((size_t)C * 4, 16);
     p.off_bar = take((size_t)kMbWords * 8, 8);
     const size_t fixed = align_up(off, 128);
@@ -927,8 +869,9 @@ bool ring_plan(int N, int HW, int C, int R, int k, int G, bool bulk_y, RingPlan 
 }  // namespace
 
 bool ring_supported(int N, int HW, int C, int R, int k) {
+    (void)N;
     RingPlan plan;
-    return ring_plan(N, HW, C, R, k, sm_count(), false, &plan);
+    return HW >= 1 && ring_plan(C, R, k, false, &plan);
 }
 
 cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
@@ -937,12 +880,66 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
                         float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
                         cudaStream_t s) {
     const int G = sm_count();
+    if (G < 1) return cudaErrorInvalidDevice;
     // every output tile [np][R + 1] starts and ends on a 16-byte boundary of y
     // when HW * (R + 1) is a multiple of 8: it leaves by one bulk copy
     const bool bulk_y =
         ((long long)HW * (R + 1)) % 8 == 0 && (reinterpret_cast<uintptr_t>(y) & 15u) == 0;
     RingPlan plan;
-    if (!ring_plan(N, HW, C, R, k, G, bulk_y, &plan)) return cudaErrorNotSupported;
+    if (!ring_plan(C, R, k, bulk_y, &plan)) return cudaErrorNotSupported;
+    const int T = (HW + kTP - 1) / kTP;
+    const unsigned long long items = (unsigned long long)N * T;
+    if (items >= 0xffff0000ull) return cudaErrorInvalidValue;
+
+    // pass 1: pooling and gate
+    PoolParams Q;
+    Q.x = x;
+    Q.N = N;
+    Q.HW = HW;
+    Q.C = C;
+    Q.R = R;
+    Q.k = k;
+    Q.T = T;
+    Q.pidx = pidx;
+    Q.plog = plog;
+    Q.W1 = W1;
+    Q.b1 = b1;
+    Q.w2 = w2;
+    Q.b2 = b2;
+    Q.tmin = tmin;
+    Q.tmax = tmax;
+    Q.ctrl = reinterpret_cast<uint32_t *>(ws + L.ctrl);
+    Q.part = reinterpret_cast<unsigned long long *>(ws + L.partial);
+    Q.zacc = reinterpret_cast<unsigned long long *>(ws + L.zacc);
+    Q.count = reinterpret_cast<uint32_t *>(ws + L.sync);
+    Q.made = Q.count + N;
+    Q.wts = reinterpret_cast<float4 *>(ws + L.a);
+    Q.z = reinterpret_cast<float *>(ws + L.z);
+    Q.tau = reinterpret_cast<float *>(ws + L.tau);
+    Q.kp = plan.kp;
+    Q.Kg = plan.Kg;
+    int per_sm = 0;
+    cudaError_t err =
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, moce_poolgate_kernel, kPoolT, 0);
+    if (err != cudaSuccess) return err;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    // runs of RL tiles: about one resident wave of CTAs, at most 255 runs per
+    // example (8-bit run counts in the accumulator words)
+    {
+        const long long slots = (long long)G * std::min(per_sm, kPoolCTAs);
+        long long rpe = std::max<long long>(1, slots / std::max(1, N));  // runs fit one wave
+        rpe = std::min<long long>(rpe, std::min<long long>(T, 255));
+        Q.RL = (int)((T + rpe - 1) / rpe);
+        Q.RPE = (T + Q.RL - 1) / Q.RL;
+        Q.runs = (uint32_t)((unsigned long long)N * Q.RPE);
+    }
+    const unsigned long long g1 =
+        std::min<unsigned long long>(Q.runs, (unsigned long long)G * std::min(per_sm, kPoolCTAs));
+    moce_poolgate_kernel<<<(unsigned)g1, kPoolT, 0, s>>>(Q);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+
+    // pass 2: mixing
     RingParams P;
     P.x = x;
     P.y = y;
@@ -952,66 +949,34 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     P.R = R;
     P.k = k;
     P.nU = nU;
-    P.T = (HW + kTP - 1) / kTP;
-    const unsigned long long items = (unsigned long long)N * P.T;
-    if (items >= 0xffff0000ull) return cudaErrorInvalidValue;
+    P.T = T;
     P.items = (uint32_t)items;
     P.pidx = pidx;
-    P.plog = plog;
     P.resid = resid;
-    P.W1 = W1;
-    P.b1 = b1;
-    P.w2 = w2;
-    P.b2 = b2;
-    P.tmin = tmin;
-    P.tmax = tmax;
-    P.ctrl = reinterpret_cast<uint32_t *>(ws + L.ctrl);
-    P.part = reinterpret_cast<float *>(ws + L.partial);
-    P.zacc = reinterpret_cast<unsigned long long *>(ws + L.zacc);
-    P.count = reinterpret_cast<uint32_t *>(ws + L.sync);
-    P.ovf = P.count + 2 * (size_t)N;
-    P.gate_tabs = plan.gate_tabs ? 1 : 0;
-    P.fix_max = 274877906944.0f / (float)P.T;  // 2^38 / T
-    P.z = reinterpret_cast<float *>(ws + L.z);
-    P.tau = reinterpret_cast<float *>(ws + L.tau);
+    P.ctrl = Q.ctrl;
+    P.wts = Q.wts;
+    P.made = Q.made;
     P.D = plan.D;
     P.CG = plan.CG;
-    P.nrow = plan.nrow;
     P.kp = plan.kp;
     P.Es = plan.Es;
-    P.ks = plan.ks;
-    P.Kg = plan.Kg;
-    P.RS = plan.RS;
     P.bulk_y = bulk_y ? 1 : 0;
     P.off_xs = (uint32_t)plan.off_xs;
     P.xs_bytes = (uint32_t)plan.xs_bytes;
     for (int b = 0; b < kNT; ++b) P.off_tab[b] = (uint32_t)plan.off_tab[b];
     for (int b = 0; b < kYB; ++b) P.off_ys[b] = (uint32_t)plan.off_ys[b];
-    P.off_rp = (uint32_t)plan.off_rp;
-    P.off_red = (uint32_t)plan.off_red;
-    P.off_zs = (uint32_t)plan.off_zs;
-    P.off_pidx = (uint32_t)plan.off_pidx;
-    P.off_plog = (uint32_t)plan.off_plog;
-    P.off_uw = (uint32_t)plan.off_uw;
-    P.off_W1 = (uint32_t)plan.off_W1;
-    P.off_b1 = (uint32_t)plan.off_b1;
-    P.off_w2 = (uint32_t)plan.off_w2;
+    P.off_res = (uint32_t)plan.off_res;
+    P.off_rred = (uint32_t)plan.off_rred;
+    P.inv_nU = nU > 0 ? 1.0f / (float)nU : 0.0f;
     P.off_U = (uint32_t)plan.off_U;
     P.off_bar = (uint32_t)plan.off_bar;
     P.inv_E = 1.0f / (float)(R + 1);
-
-    cudaError_t err = cudaFuncSetAttribute(moce_ring_kernel,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)plan.smem);
-    if (err != cudaSuccess) return err;
-    int per_sm = 0;
-    if ((err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, moce_ring_kernel, kRingT,
-                                                             plan.smem)) != cudaSuccess)
+    if ((err = cudaFuncSetAttribute(moce_ring_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)plan.smem)) != cudaSuccess)
         return err;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    void *args[] = {&P};
-    return cudaLaunchCooperativeKernel((const void *)moce_ring_kernel, dim3(G), dim3(kRingT), args,
-                                       plan.smem, s);
+    const unsigned g2 = (unsigned)std::min<unsigned long long>(items, (unsigned long long)G);
+    moce_ring_kernel<<<g2, kRingT, plan.smem, s>>>(P);
+    return cudaGetLastError();
 }
 
 }  // namespace moce

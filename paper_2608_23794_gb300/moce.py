@@ -61,6 +61,10 @@ def library():
             "moce_pool": ([P, I, I, I, I, I, I, P, P, S, P], I),
             "moce_gate": ([P, I, I, I, I, P, P, P, P, P, P, F, F, P, P, P], I),
             "moce_forward": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S, P], I),
+            "moce_forward_path": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, S,
+                                   I, P], I),
+            "moce_forward_path_launches": ([P, I, I, I, I, I, I, I, I, I], I),
+            "moce_forward_path_kernel": ([P, I, I, I, I, I, I, I, I, I], ctypes.c_char_p),
             "moce_check_device_error": ([P, S, P], I),
             "moce_forward_launches": ([P, I, I, I, I, I, I, I, I], I),
             "moce_forward_kernel": ([P, I, I, I, I, I, I, I, I], ctypes.c_char_p),
@@ -208,9 +212,14 @@ def moce_gate(z: torch.Tensor, packed: PackedSupports, W1, b1, w2, b2, tau_min: 
     return tau, a
 
 
+# moce_path_t: the kernel path of one forward (AUTO = the fastest that fits)
+PATHS = {"auto": 0, "pipe": 1, "two_pass": 2, "fused": 3, "steps": 4}
+
+
 def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
                  tau_min: float, tau_max: float, ws: Workspace | None = None,
-                 y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+                 y: torch.Tensor | None = None, stream=None, path: str = "auto") -> torch.Tensor:
+    """The layer forward (Sec. 3.2-3.4); ``path`` forces one kernel path (``PATHS``)."""
     N, H, W, C = _dims(x, layout)
     R, k = packed.C_out, packed.k
     if C != packed.C_in:
@@ -220,25 +229,38 @@ def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w
         y = torch.empty(shape, dtype=x.dtype, device=x.device)
     if ws is None:
         ws = Workspace(N, H, W, C, R, k, device=x.device)
-    _check(library().moce_forward(_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout],
-                                  _ptr(packed.packed_idx), _ptr(packed.packed_logits),
-                                  _ptr(packed.resid_idx), packed.n_resid, _ptr(W1), _ptr(b1),
-                                  _ptr(w2), _ptr(b2), float(tau_min), float(tau_max), _ptr(y),
-                                  _ptr(ws.buffer), ws.nbytes, _stream(stream)), "moce_forward")
+    lib = library()
+    args = (_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout], _ptr(packed.packed_idx),
+            _ptr(packed.packed_logits), _ptr(packed.resid_idx), packed.n_resid, _ptr(W1), _ptr(b1),
+            _ptr(w2), _ptr(b2), float(tau_min), float(tau_max), _ptr(y), _ptr(ws.buffer), ws.nbytes)
+    if path == "auto":
+        _check(lib.moce_forward(*args, _stream(stream)), "moce_forward")
+    else:
+        _check(lib.moce_forward_path(*args, PATHS[path], _stream(stream)), "moce_forward_path")
     return y
 
 
-def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int) -> int:
-    """Kernel launches one moce_forward call makes for this input."""
+def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int,
+                          path: str = "auto") -> int:
+    """Kernel launches one moce_forward call makes for this input (0: path cannot run it)."""
     N, H, W, C = _dims(x, layout)
-    return int(library().moce_forward_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
-                                                _LAYOUTS[layout]))
+    if path == "auto":
+        return int(library().moce_forward_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
+                                                    _LAYOUTS[layout]))
+    return int(library().moce_forward_path_launches(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
+                                                     _LAYOUTS[layout], PATHS[path]))
 
 
-def moce_forward_kernel(x: torch.Tensor, layout: str, C_out: int, k: int) -> str:
+def moce_forward_kernel(x: torch.Tensor, layout: str, C_out: int, k: int,
+                        path: str = "auto") -> str:
     """Name of the kernel path one moce_forward call takes for this input."""
     N, H, W, C = _dims(x, layout)
-    name = library().moce_forward_kernel(_ptr(x), N, H, W, C, C_out, k, _dtype(x), _LAYOUTS[layout])
+    if path == "auto":
+        name = library().moce_forward_kernel(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
+                                             _LAYOUTS[layout])
+    else:
+        name = library().moce_forward_path_kernel(_ptr(x), N, H, W, C, C_out, k, _dtype(x),
+                                                  _LAYOUTS[layout], PATHS[path])
     if name is None:
         raise MoceError(1, "moce_forward_kernel")
     return name.decode()

@@ -31,7 +31,7 @@ def device_tensors(lay: synth.SyntheticLayer, device="cuda"):
     )
 
 
-def gpu_forward(lay: synth.SyntheticLayer, dev=None, ws=None):
+def gpu_forward(lay: synth.SyntheticLayer, dev=None, ws=None, path="auto"):
     """Returns (y float64 numpy, packed, ws) from moce_pack_supports + moce_forward."""
     import torch
     from paper_2608_23794_gb300 import moce
@@ -41,7 +41,7 @@ def gpu_forward(lay: synth.SyntheticLayer, dev=None, ws=None):
     if ws is None:
         ws = moce.Workspace(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k)
     y = moce.moce_forward(dev["x"], cfg.layout, packed, dev["W1"], dev["b1"], dev["w2"], dev["b2"],
-                          cfg.tau_min, cfg.tau_max, ws=ws)
+                          cfg.tau_min, cfg.tau_max, ws=ws, path=path)
     torch.cuda.synchronize()
     moce.moce_check_device_error(ws)
     return y.float().cpu().numpy().astype(np.float64), packed, ws

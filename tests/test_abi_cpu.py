@@ -87,6 +87,46 @@ def test_forward_rejects_bad_arguments_on_host(lib):
     assert call(N=0) == 0  # empty batch: nothing to do
 
 
+def test_forward_path_selection_on_host(lib):
+    P, I, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    f = lib.moce_forward_path
+    f.argtypes = [P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P, ctypes.c_size_t,
+                  I, P]
+    f.restype = I
+    n = lib.moce_forward_path_launches
+    n.argtypes = [P, I, I, I, I, I, I, I, I, I]
+    n.restype = I
+    name = lib.moce_forward_path_kernel
+    name.argtypes = n.argtypes
+    name.restype = ctypes.c_char_p
+    fake = ctypes.c_void_p(0x1000)  # 256-byte aligned, never dereferenced
+
+    def call(dt, path, ws_bytes=1 << 40):
+        return f(fake, 2, 8, 8, 64, 16, 4, dt, 0, fake, fake, fake, 3, fake, fake, fake, fake,
+                 0.2, 6.0, fake, fake, ws_bytes, path, None)
+
+    assert call(1, 7) == 1             # not a path
+    assert call(1, -1) == 1
+    assert call(0, 2) == 3             # fp32 has no two-pass kernel: unsupported, nothing enqueued
+    assert call(0, 1) == 3             # nor a pipeline kernel
+    # bf16 NHWC, aligned x: every path runs these shapes
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 1
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"moce_pipe_kernel"
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == 2
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == b"moce_poolgate_kernel+moce_ring_kernel"
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 3) == 1
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == b"pool+gate+mix"
+    # misaligned x or NCHW leaves only the step kernels
+    odd = ctypes.c_void_p(0x1002)
+    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 1) == 0
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 2) == 0
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3
+    # more experts than the two-pass kernel's pairs
+    assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 2) == 0
+    assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 1) == 1
+
+
 def test_pack_rejects_bad_arguments_on_host(lib):
     f = lib.moce_pack_supports
     P, I = ctypes.c_void_p, ctypes.c_int

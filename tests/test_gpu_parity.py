@@ -250,3 +250,49 @@ def test_forward_full_size_sampled(name):
     assert np.isfinite(y).all()
     z = ws.z().cpu().numpy()
     np.testing.assert_allclose(z[ex], oracle.pool(lay.x[ex], cfg.layout), rtol=1e-5, atol=1e-6)
+
+
+# ------------------------------------------------------------------ every kernel path
+
+
+PATHS = ["pipe", "two_pass", "fused", "steps"]
+PATH_CASES = {
+    "rn50_stage1_reduce": SMALL["rn50_stage1_reduce"],
+    "c72_r9_k5": EDGE["c72_r9_k5"],
+    "k1": EDGE["k1"],
+    "k_eq_c": EDGE["k_eq_c"],
+    "hw1": EDGE["hw1"],
+    "r3": EDGE["r3"],
+    "f32_nhwc": EDGE["f32_nhwc"],
+}
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("name", list(PATH_CASES))
+def test_every_path_matches_oracle(name, path):
+    from paper_2608_23794_gb300 import moce
+    cfg = PATH_CASES[name]
+    lay = synth.make_layer(cfg, seed=3)
+    dev = device_tensors(lay)
+    if moce.moce_forward_launches(dev["x"], cfg.layout, cfg.C_out, cfg.k, path=path) == 0:
+        with pytest.raises(moce.MoceError):
+            gpu_forward(lay, dev=dev, path=path)
+        return
+    y1, _, ws = gpu_forward(lay, dev=dev, path=path)
+    assert_close(y1, oracle_forward(lay), cfg.dtype)
+    # a second call on the same workspace gives the same bits
+    y2, _, _ = gpu_forward(lay, dev=dev, ws=ws, path=path)
+    assert np.array_equal(y1, y2)
+
+
+@pytest.mark.parametrize("path", ["pipe", "two_pass"])
+def test_stage1_full_size_every_path(path):
+    from paper_2608_23794_gb300 import moce
+    cfg = CFG["rn50_stage1_reduce"]
+    lay = synth.make_layer(cfg, seed=5)
+    dev = device_tensors(lay)
+    assert moce.moce_forward_launches(dev["x"], cfg.layout, cfg.C_out, cfg.k, path=path) >= 1
+    y, _, _ = gpu_forward(lay, dev=dev, path=path)
+    ex = [1, cfg.N // 3, cfg.N - 2]
+    assert_close(y[ex], oracle_forward(lay, examples=ex), cfg.dtype)
+    assert np.isfinite(y).all()
