@@ -18,21 +18,25 @@
 //
 // Mixing table: for expert pair p (experts 2p, 2p + 1) and support positions
 // (2 i2, 2 i2 + 1), one float4 {w(2p, 2i2), w(2p, 2i2+1), w(2p+1, 2i2),
-// w(2p+1, 2i2+1)} at entry [p][i2 ^ ((p >> 3) & 3)] of a [32][8] block: the
+// w(2p+1, 2i2+1)} at entry [i2][4 (p mod 8) + p / 8] of an [8][32] block: a
+// mixing lane reads its pair's entries 512 bytes apart from one base, and the
 // four lane groups of a mixing warp (pairs 8 apart) read different banks.
 //
 // Pass 2, moce_ring_kernel, reads x again and mixes it: one CTA per SM takes
-// items b, b + G, ...; its load warps (8-23) stage each tile, transposed to
-// channel-major rows, into a ring of D shared-memory slots two tiles ahead;
-// the table warps (24-27) copy the item's weights into one of three mixing
-// tables and sum the tile's unselected channels for the residual expert
-// (Eq. (res)); the mix warps (0-7) mix a slot with its table: each group of 8
-// lanes owns 8 positions per lane and one expert pair for the whole launch,
-// whose row offsets it keeps in registers (Eq. (expert)); the tile of y,
-// residual column included, leaves by one bulk copy. The
-// roles hand slots and tables over through shared-memory mbarriers (one
-// thread waits, the others block at a barrier); every wait is bounded and
-// none crosses CTAs.
+// items b, b + G, ...; its copy warp (19) brings each tile (64 positions x C
+// channels, contiguous in NHWC) into a ring of D shared-memory slots by one
+// bulk copy as soon as a slot is free, so several tiles are in flight; the
+// load warps (8-15) transpose a landed tile in place to channel-major rows;
+// the table warps (16-18) bring the weights of the item two ahead into one of
+// four mixing tables by a bulk copy and sum the tile's unselected channels
+// for the residual expert (Eq. (res)); the mix warps (0-7) mix a slot with
+// its table: each group of 8 lanes owns 8 positions per lane and one expert
+// pair for the whole launch, whose row offsets it keeps in registers
+// (Eq. (expert)); the tile of y, residual column included, leaves by one bulk
+// copy. The roles hand slots and tables over through shared-memory
+// mbarriers; every wait is bounded and none crosses CTAs. No role holds
+// global loads in registers across a barrier: x and the weights arrive by
+// bulk copies, so the barriers never wait for HBM.
 #include <algorithm>
 
 #include "moce_device.cuh"
@@ -44,15 +48,19 @@ constexpr int kTP = kRingTile;        // positions per tile
 constexpr int kGS = 8;                // lanes of a mixing group
 constexpr int kRB = 16 * kGS;         // bytes per staged channel row (kTP bf16)
 constexpr int kFM = 7;                // chunk swizzle mask of the staged rows
-constexpr int kMixT = 256;            // pass 2: mix warps 0-7
-constexpr int kLoadT = 512;           // pass 2: load warps 8-23
-constexpr int kTabT = 128;            // pass 2: table warps 24-27
-constexpr int kRingT = kMixT + kLoadT + kTabT;
+constexpr int kMixT = 512;            // pass 2: mix warps 0-15
+constexpr int kLoadT = 256;           // pass 2: load warps 16-23
+constexpr int kTabT = 96;             // pass 2: table warps 24-26
+constexpr int kProdT = 32;            // pass 2: the copy warp 27
+constexpr int kLoadW = kLoadT / 32;
+constexpr int kLU = 32 / kLoadW;      // staging units per load thread and tile (at C = 256)
+constexpr int kRingT = kMixT + kLoadT + kTabT + kProdT;
 constexpr int kLoad0 = kMixT;                    // first load thread
 constexpr int kTab0 = kMixT + kLoadT;            // first table thread
+constexpr int kProd0 = kTab0 + kTabT;            // the copy warp's first thread
 constexpr int kResParts = kTabT / 8;             // residual: U entries split kResParts ways
-constexpr int kMixWarps = kMixT / 32;
-constexpr int kNT = 3;                // mixing tables
+constexpr int kPairWarps = 8;         // mix warps w and w + 8 share expert pairs
+constexpr int kNT = 4;                // mixing tables (weights arrive two items ahead)
 constexpr int kYB = 2;                // output tile buffers
 constexpr int kRS = 4;                // residual columns (the table role runs ahead)
 constexpr int kMaxD = 6;              // x slots at most
@@ -60,18 +68,18 @@ constexpr int kGateMaxK = 16;          // support positions a mixing lane keeps 
 constexpr int kMaxPairs = 32;          // expert pairs: one per mixing group
 constexpr int kWBlock = kMaxPairs * 8; // float4 entries of a weight block
 constexpr int kBarMix = 1, kBarLoad = 2, kBarTab = 3;
-// Registers per thread: the launch gives every thread 72 (kRingT * 72 <=
-// 65536); the roles then trade them with setmaxnreg within that total (the
-// mixing loop keeps its row offsets in registers).
-constexpr int kLaunchRegs = 72, kMixRegs = 96, kLoadRegs = 64, kTabRegs = 56;
-static_assert(kMixT * kMixRegs + kLoadT * kLoadRegs + kTabT * kTabRegs <= kRingT * kLaunchRegs,
+// Registers per thread: 72 for every role (kRingT * 72 <= 65536).
+constexpr int kLaunchRegs = 72, kMixRegs = 72, kLoadRegs = 72, kTabRegs = 72;
+static_assert(kMixT * kMixRegs + kLoadT * kLoadRegs + (kTabT + kProdT) * kTabRegs <=
+                  kRingT * kLaunchRegs,
               "register split exceeds the launch allocation");
-static_assert(kMixT % 128 == 0 && kLoadT % 128 == 0 && kTabT % 128 == 0, "whole warpgroups");
+static_assert(kMixT % 128 == 0 && kLoadT % 128 == 0 && (kTabT + kProdT) % 128 == 0,
+              "whole warpgroups (the copy warp shares the table warps' register count)");
 constexpr int kPoolT = 256;           // pass 1 threads per CTA
 constexpr int kPoolCTAs = 8;          // pass 1 CTAs per SM
 constexpr int kAccG = 4;              // accumulator words per (example, channel)
 static_assert(kRingT * kLaunchRegs <= 65536, "launch registers at one CTA per SM");
-static_assert(kMixT == 4 * kTP, "four mixing threads per position in the epilogue");
+static_assert(kMixT == 2 * kPairWarps * 32, "two mix warps per set of expert pairs");
 static_assert(kTP == 8 * kGS, "a group's lanes cover the tile");
 static_assert(kPoolT == 4 * kTP, "pass 1: 32 channel blocks x 8 rows of positions");
 
@@ -86,17 +94,18 @@ constexpr float kFixMax = 524288.0f;     // 2^19
 constexpr unsigned long long kFixBias = 1ull << 39;
 constexpr unsigned long long kWideOne = 1ull << 48;
 
-// mbarriers of pass 2 (8 bytes each): full[s] (load -> mix, table), empty[s]
-// (mix and table -> load: two arrivals), tready[b] (table -> mix), tfree[b]
-// (mix -> table), rdone[c] (table -> mix: residual column c), rfree[c]
-// (mix -> table).
+// mbarriers of pass 2 (8 bytes each): raw[s] (the bulk copy of a tile into
+// slot s has landed: copy warp's arrival + transaction bytes), full[s]
+// (load -> mix, table), empty[s] (mix and table -> copy warp: two
+// arrivals), tready[b] (table -> mix), tfree[b] (mix -> table), rdone[c]
+// (table -> mix: residual column c), rfree[c] (mix -> table).
 constexpr int kMbFull = 0, kMbEmpty = kMaxD, kMbTReady = 2 * kMaxD, kMbTFree = 2 * kMaxD + kNT,
               kMbRDone = 2 * kMaxD + 2 * kNT, kMbRFree = 2 * kMaxD + 2 * kNT + kRS,
-              kMbWords = 2 * kMaxD + 2 * kNT + 2 * kRS;
+              kMbRaw = 2 * kMaxD + 2 * kNT + 2 * kRS, kMbWords = 3 * kMaxD + 2 * kNT + 2 * kRS;
 
 // float4 entry of expert pair p, support positions (2 i2, 2 i2 + 1), in a
 // weight block.
-__device__ __forceinline__ int wslot(int p, int i2) { return p * 8 + (i2 ^ ((p >> 3) & 3)); }
+__device__ __forceinline__ int wslot(int p, int i2) { return i2 * 32 + 4 * (p & 7) + (p >> 3); }
 
 struct PoolParams {
     const uint16_t *x;
@@ -122,6 +131,7 @@ struct RingParams {
     uint16_t *y;
     int N, HW, C, R, k, nU, T;
     uint32_t items;               // N * T tiles
+    int Gn, Gt;                   // the grid size G = Gn * T + Gt (items a CTA steps over)
     const int32_t *pidx;
     const int32_t *resid;
     uint32_t *ctrl;
@@ -404,15 +414,15 @@ __global__ void __launch_bounds__(kPoolT) moce_poolgate_kernel(const PoolParams 
 // pixel pairs into rows 8 cc .. 8 cc + 7, word j of chunk q ^ (cc & 7). A
 // mixing lane that reads chunk q of a row gets positions q + 8 m, m = 0..7.
 // Lane l of load warp w: cc = 8 (w mod CG) + (l mod 8), j = l / 8, units
-// q = (w + 16 i) / CG for i = 0, 1 while w + 16 i < 8 CG; a warp's loads
-// read 128 contiguous bytes per position and its stores hit 32 banks.
+// q = (w + 8 i) / CG for i = 0 .. kLU - 1 while w + 8 i < 8 CG; a warp's
+// reads take 128 contiguous bytes per position and its stores hit 32 banks.
 struct LoadUnits {
-    int nu;          // units per tile (0..2)
+    int nu;          // units per tile (0..kLU)
     int cc;          // 8-channel block
     bool own;        // cc < C / 8
-    int pa[2];       // low position of each unit (the high one is pa + 8)
-    int src[2];      // element offset of the low position's load in a tile of x
-    int dst[2];      // byte offset of the unit's first word in a slot
+    int pa[kLU];     // low position of each unit (the high one is pa + 8)
+    int src[kLU];    // element offset of the low position in a tile of x
+    int dst[kLU];    // byte offset of the unit's first word in a slot
 };
 
 __device__ __forceinline__ LoadUnits load_units(const RingParams &P, int lt) {
@@ -421,10 +431,12 @@ __device__ __forceinline__ LoadUnits load_units(const RingParams &P, int lt) {
     const int j = lane >> 3;
     u.cc = 8 * (w & (P.CG - 1)) + (lane & 7);
     u.own = u.cc < (P.C >> 3);
-    u.nu = (w < 8 * P.CG) + (w + 16 < 8 * P.CG);
+    u.nu = 0;
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const int q = (w + 16 * i) / P.CG;
+    for (int i = 0; i < kLU; ++i) u.nu += (w + kLoadW * i < 8 * P.CG);
+#pragma unroll
+    for (int i = 0; i < kLU; ++i) {
+        const int q = (w + kLoadW * i) / P.CG;
         u.pa[i] = q + 16 * j;
         u.src[i] = u.pa[i] * P.C + u.cc * 8;
         u.dst[i] = (u.cc * 8) * kRB + (((q ^ (u.cc & kFM)) << 4) | (j << 2));
@@ -432,74 +444,116 @@ __device__ __forceinline__ LoadUnits load_units(const RingParams &P, int lt) {
     return u;
 }
 
-// The loads of item it (none past the last item; positions past the end of
-// the example read nothing).
-__device__ __forceinline__ void tile_loads(const RingParams &P, const LoadUnits &u, uint32_t it,
-                                           uint4 *v) {
-    const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
-    if (it >= P.items) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) v[i] = zero;
-        return;
+// A role's position in its items b, b + G, ...: round r, item it (example n,
+// tile t), slot s = r mod D and its phase bit (r / D) mod 2, advanced
+// without divisions.
+struct Round {
+    uint32_t r, it, s, ph;
+    int n, t;
+    __device__ __forceinline__ explicit Round(const RingParams &P)
+        : r(0), it(blockIdx.x), s(0), ph(0) {
+        n = (int)(blockIdx.x / (uint32_t)P.T);
+        t = (int)blockIdx.x - n * P.T;
     }
-    const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
-    const int p0 = t * kTP, np = min(kTP, P.HW - p0);
-    const uint16_t *xt = P.x + ((size_t)n * P.HW + p0) * P.C;
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const bool on = i < u.nu && u.own;
-        v[2 * i] = (on && u.pa[i] < np) ? ld_stream(xt + u.src[i]) : zero;
-        v[2 * i + 1] = (on && u.pa[i] + 8 < np) ? ld_stream(xt + u.src[i] + 8 * P.C) : zero;
+    __device__ __forceinline__ bool live(const RingParams &P) const { return it < P.items; }
+    __device__ __forceinline__ void next(const RingParams &P) {
+        ++r;
+        it += gridDim.x;
+        if (++s == (uint32_t)P.D) {
+            s = 0;
+            ph ^= 1u;
+        }
+        n += P.Gn;
+        t += P.Gt;
+        if (t >= P.T) {
+            t -= P.T;
+            ++n;
+        }
     }
+    __device__ __forceinline__ int p0() const { return t * kTP; }
+    __device__ __forceinline__ int np(const RingParams &P) const { return min(kTP, P.HW - t * kTP); }
+};
+
+// The copy warp: one bulk copy per item of the tile's np * C contiguous bf16
+// (NHWC) into slot r mod D, once the mix and table roles have released the
+// slot; raw[s] completes when the bytes have landed. On a wait that gave up,
+// the copies still in flight land before the warp returns.
+__device__ void copy_role(const RingParams &P, unsigned char *sm) {
+    set_role_regs<kTabRegs, kLaunchRegs>();
+    if ((threadIdx.x & 31) == 0) {
+        Round q(P);
+        bool ok = true;
+        for (; q.live(P); q.next(P)) {
+            if (q.r >= (uint32_t)P.D &&
+                !ring_wait(mbar(P, sm, kMbEmpty + q.s), q.ph ^ 1u, P.ctrl, q.it)) {
+                ok = false;
+                break;
+            }
+            const uint32_t bytes = (uint32_t)q.np(P) * (uint32_t)P.C * 2u;
+            const uint16_t *src = P.x + ((size_t)q.n * P.HW + q.p0()) * P.C;
+            const uint32_t s = q.s;
+            const uint32_t bar = mbar(P, sm, kMbRaw + s);
+            // the slot's earlier generic-proxy reads and writes come before the copy
+            asm volatile(
+                "fence.proxy.async.shared::cta;\n\t"
+                "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, "
+                "[%0];" ::"r"(bar),
+                "r"(bytes), "r"(smem_u32(sm + P.off_xs + s * P.xs_bytes)), "l"(src)
+                : "memory");
+        }
+        if (!ok) {
+            const uint32_t r = q.r;
+            for (uint32_t j = r > (uint32_t)P.D ? r - (uint32_t)P.D : 0u; j < r; ++j) {
+                const uint32_t bar = mbar(P, sm, kMbRaw + j % (uint32_t)P.D);
+                for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (j / P.D) & 1u); ++i)
+                    __nanosleep(256);
+            }
+        }
+    }
+    __syncwarp();
 }
 
-// One item of the load role: store the tile held in v into slot r mod D and
-// refill v with the loads of the item two ahead. False when a wait gave up.
-__device__ __forceinline__ bool load_item(const RingParams &P, unsigned char *sm,
-                                          const LoadUnits &u, uint32_t it, uint32_t r, uint4 *v) {
-    const int lt = threadIdx.x - kLoad0;
-    const uint32_t s = r % (uint32_t)P.D;
-    // slot s is free once the mix role is done with item r - D
-    bool ok = true;
-    if (lt == 0 && r >= (uint32_t)P.D)
-        ok = ring_wait(mbar(P, sm, kMbEmpty + s), ((r / P.D) - 1u) & 1u, P.ctrl, it);
-    if (!bar_and(kBarLoad, kLoadT, ok)) return false;
-    unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        if (i >= u.nu || !u.own) continue;
-        unsigned char *d = xs + u.dst[i];
-        const uint4 va = v[2 * i], vb = v[2 * i + 1];
-        *reinterpret_cast<uint32_t *>(d + 0 * kRB) = __byte_perm(va.x, vb.x, 0x5410);
-        *reinterpret_cast<uint32_t *>(d + 1 * kRB) = __byte_perm(va.x, vb.x, 0x7632);
-        *reinterpret_cast<uint32_t *>(d + 2 * kRB) = __byte_perm(va.y, vb.y, 0x5410);
-        *reinterpret_cast<uint32_t *>(d + 3 * kRB) = __byte_perm(va.y, vb.y, 0x7632);
-        *reinterpret_cast<uint32_t *>(d + 4 * kRB) = __byte_perm(va.z, vb.z, 0x5410);
-        *reinterpret_cast<uint32_t *>(d + 5 * kRB) = __byte_perm(va.z, vb.z, 0x7632);
-        *reinterpret_cast<uint32_t *>(d + 6 * kRB) = __byte_perm(va.w, vb.w, 0x5410);
-        *reinterpret_cast<uint32_t *>(d + 7 * kRB) = __byte_perm(va.w, vb.w, 0x7632);
-    }
-    // the item two ahead is in flight while the next one is stored
-    tile_loads(P, u, it + 2u * gridDim.x, v);
-    bar_sync(kBarLoad, kLoadT);
-    if (lt == 0) mbar_arrive(mbar(P, sm, kMbFull + s));
-    return true;
-}
-
-// Items alternate between the two register sets (unrolled by two, so each
-// set stays in registers).
-__device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnits &u, uint4 *va,
-                          uint4 *vb) {
+// The load role, per item r: once raw[s] completes, every thread reads its
+// staging units of the raw tile in slot s (positions past np read as 0),
+// the role meets at a barrier, and the units are written back in place as
+// channel-major rows of pixel pairs (the raw tile, np * C * 2 bytes, lies
+// within rows 0 .. C - 1, so row C stays zero).
+__device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnits &u) {
     set_role_regs<kLoadRegs, kLaunchRegs>();
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items;) {
-        if (!load_item(P, sm, u, it, r, va)) break;
-        it += gridDim.x;
-        ++r;
-        if (it >= P.items) break;
-        if (!load_item(P, sm, u, it, r, vb)) break;
-        it += gridDim.x;
-        ++r;
+    const int lt = threadIdx.x - kLoad0;
+    const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+    for (Round q(P); q.live(P); q.next(P)) {
+        const uint32_t s = q.s;
+        bool ok = true;
+        if (lt == 0) ok = ring_wait(mbar(P, sm, kMbRaw + s), q.ph, P.ctrl, q.it);
+        if (!bar_and(kBarLoad, kLoadT, ok)) return;
+        const int np = q.np(P);
+        unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
+        uint4 v[2 * kLU];
+#pragma unroll
+        for (int i = 0; i < kLU; ++i) {
+            const bool on = i < u.nu && u.own;
+            v[2 * i] = (on && u.pa[i] < np) ? lds128(xs + 2 * u.src[i]) : zero;
+            v[2 * i + 1] = (on && u.pa[i] + 8 < np) ? lds128(xs + 2 * (u.src[i] + 8 * P.C)) : zero;
+        }
+        bar_sync(kBarLoad, kLoadT);  // the raw tile is read
+#pragma unroll
+        for (int i = 0; i < kLU; ++i) {
+            if (i >= u.nu || !u.own) continue;
+            unsigned char *d = xs + u.dst[i];
+            const uint4 va = v[2 * i], vb = v[2 * i + 1];
+            *reinterpret_cast<uint32_t *>(d + 0 * kRB) = __byte_perm(va.x, vb.x, 0x5410);
+            *reinterpret_cast<uint32_t *>(d + 1 * kRB) = __byte_perm(va.x, vb.x, 0x7632);
+            *reinterpret_cast<uint32_t *>(d + 2 * kRB) = __byte_perm(va.y, vb.y, 0x5410);
+            *reinterpret_cast<uint32_t *>(d + 3 * kRB) = __byte_perm(va.y, vb.y, 0x7632);
+            *reinterpret_cast<uint32_t *>(d + 4 * kRB) = __byte_perm(va.z, vb.z, 0x5410);
+            *reinterpret_cast<uint32_t *>(d + 5 * kRB) = __byte_perm(va.z, vb.z, 0x7632);
+            *reinterpret_cast<uint32_t *>(d + 6 * kRB) = __byte_perm(va.w, vb.w, 0x5410);
+            *reinterpret_cast<uint32_t *>(d + 7 * kRB) = __byte_perm(va.w, vb.w, 0x7632);
+        }
+        bar_sync(kBarLoad, kLoadT);
+        if (lt == 0) mbar_arrive(mbar(P, sm, kMbFull + s));
     }
 }
 
@@ -510,6 +564,23 @@ __device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnit
 // (Eq. (res)): thread (q = chunk, part) adds U entries part, part +
 // kResParts, ... for the chunk's 8 positions, the parts are added in order,
 // and res[r mod kYB][p] = sum / |U| (0 if U is empty).
+// One bulk copy of the weight block of round q's example into table
+// q.r mod kNT; tready of that table completes when the 4 KB have landed.
+__device__ __forceinline__ void weights_copy(const RingParams &P, unsigned char *sm,
+                                             const Round &q) {
+    const uint32_t tb = q.r % kNT;
+    const uint32_t bar = mbar(P, sm, kMbTReady + tb);
+    // the mix role's reads of the table's previous contents come first
+    asm volatile(
+        "fence.proxy.async.shared::cta;\n\t"
+        "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, "
+        "[%0];" ::"r"(bar),
+        "r"((uint32_t)(kWBlock * 16)), "r"(smem_u32(sm + P.off_tab[tb])),
+        "l"(P.wts + (size_t)q.n * kWBlock)
+        : "memory");
+}
+
 __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag) {
     set_role_regs<kTabRegs, kLaunchRegs>();
     const int tt = threadIdx.x - kTab0;
@@ -517,28 +588,34 @@ __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag)
     const uint32_t lx = (uint32_t)q << 4;
     const int32_t *s_resid = reinterpret_cast<const int32_t *>(sm + P.off_U);
     float *rred = reinterpret_cast<float *>(sm + P.off_rred);
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t tb = r % kNT, s = r % (uint32_t)P.D, rc = r % kRS;
-        const int n = (int)(it / (uint32_t)P.T);
-        bool ok = true;
-        if (tt == 0 && r >= (uint32_t)kNT)
-            ok = ring_wait(mbar(P, sm, kMbTFree + tb), ((r / kNT) - 1u) & 1u, P.ctrl, it);
-        if (!bar_and(kBarTab, kTabT, ok)) break;
-        if (tt == 0 && __ldg(P.made + n) != tag) report_timeout(P.ctrl, it);
-        {
-            const float4 *wn = P.wts + (size_t)n * kWBlock;
-            float4 *tab = reinterpret_cast<float4 *>(sm + P.off_tab[tb]);
-            float4 w[kWBlock / kTabT];
-#pragma unroll
-            for (int j = 0; j < kWBlock / kTabT; ++j) w[j] = __ldg(wn + tt + kTabT * j);
-#pragma unroll
-            for (int j = 0; j < kWBlock / kTabT; ++j) tab[tt + kTabT * j] = w[j];
+    // thread 0 keeps the weights of the next two items in flight
+    Round ahead(P);
+    if (tt == 0) {
+        for (int i = 0; i < 2 && ahead.live(P); ++i) {
+            weights_copy(P, sm, ahead);
+            ahead.next(P);
         }
-        bar_sync(kBarTab, kTabT);
+    }
+    for (Round rd(P); rd.live(P); rd.next(P)) {
+        const uint32_t r = rd.r, it = rd.it, s = rd.s;
+        const uint32_t rc = r % kRS;
+        const int n = rd.n;
+        bool ok = true;
         if (tt == 0) {
-            mbar_arrive(mbar(P, sm, kMbTReady + tb));
-            ok = ring_wait(mbar(P, sm, kMbFull + s), (r / P.D) & 1u, P.ctrl, it);
+            if (__ldg(P.made + n) != tag) report_timeout(P.ctrl, it);
+            if (ahead.live(P)) {
+                // table ahead.r mod kNT is free once the mix role is done with
+                // item ahead.r - kNT
+                const uint32_t tb = ahead.r % kNT;
+                if (ahead.r >= (uint32_t)kNT)
+                    ok = ring_wait(mbar(P, sm, kMbTFree + tb), ((ahead.r / kNT) - 1u) & 1u,
+                                   P.ctrl, it);
+                if (ok) {
+                    weights_copy(P, sm, ahead);
+                    ahead.next(P);
+                }
+            }
+            if (ok) ok = ring_wait(mbar(P, sm, kMbFull + s), rd.ph, P.ctrl, it);
             if (ok && r >= (uint32_t)kRS)
                 ok = ring_wait(mbar(P, sm, kMbRFree + rc), ((r / kRS) - 1u) & 1u, P.ctrl, it);
         }
@@ -568,6 +645,16 @@ __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag)
         bar_sync(kBarTab, kTabT);  // rred is free again; the residual column is complete
         if (tt == 0) mbar_arrive(mbar(P, sm, kMbRDone + rc));
     }
+    // after a wait gave up, the weight copies still in flight land before the
+    // CTA exits (after a normal end the mix role has waited for all of them)
+    if (tt == 0 && ahead.r > 0) {
+        const uint32_t last = ahead.r;
+        for (uint32_t j = last > (uint32_t)kNT ? last - (uint32_t)kNT : 0u; j < last; ++j) {
+            const uint32_t bar = mbar(P, sm, kMbTReady + j % kNT);
+            for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (j / kNT) & 1u); ++i)
+                __nanosleep(256);
+        }
+    }
 }
 
 // ================================================================ mix role
@@ -577,41 +664,45 @@ __device__ __forceinline__ uint32_t row_off(uint32_t c, uint32_t lx) {
     return ((c * kRB) | (((c >> 3) & kFM) << 4)) ^ lx;
 }
 
-// Weighted sums of the lane's expert pair for its 8 positions: per entry i2,
-// one float4 of weights and four 16-byte row chunks whose offsets the lane
-// holds in registers (offs[2 i2]: expert a, positions 2 i2 and 2 i2 + 1, low
-// and high half; offs[2 i2 + 1]: expert b).
-__device__ __forceinline__ void mix_pair_regs(const unsigned char *xs, const float4 *wt, int pr,
-                                              int npairs, const uint32_t *offs, float2 &a0,
-                                              float2 &a1, float2 &a2, float2 &a3, float2 &b0,
-                                              float2 &b1, float2 &b2, float2 &b3) {
+// Shared-memory loads at 32-bit shared-window addresses.
+__device__ __forceinline__ uint2 lds64(uint32_t a) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ float4 lds128f(uint32_t a) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(a));
+    return v;
+}
+
+// Weighted sums of the lane's expert pair for its 4 positions: per entry i2,
+// one float4 of weights (at wa + 512 i2) and four 8-byte halves of row
+// chunks at xa + offs[4 i2 + j] (j = 0, 1: expert a, support positions 2 i2,
+// 2 i2 + 1; j = 2, 3: expert b).
+__device__ __forceinline__ void mix_pair_half(uint32_t xa, uint32_t wa, int npairs,
+                                              const uint32_t *offs, float2 &a0, float2 &a1,
+                                              float2 &b0, float2 &b1) {
 #pragma unroll
     for (int i2 = 0; i2 < kGateMaxK / 2; ++i2) {
         if (i2 >= npairs) break;
-        const float4 w = wt[wslot(pr, i2)];
-        const uint32_t oa = offs[2 * i2], ob = offs[2 * i2 + 1];
-        const uint4 va0 = lds128(xs + (oa & 0xffffu));
-        const uint4 va1 = lds128(xs + (oa >> 16));
-        const uint4 vb0 = lds128(xs + (ob & 0xffffu));
-        const uint4 vb1 = lds128(xs + (ob >> 16));
+        const float4 w = lds128f(wa + 512u * i2);
+        const uint2 va0 = lds64(xa + offs[4 * i2 + 0]);
+        const uint2 va1 = lds64(xa + offs[4 * i2 + 1]);
+        const uint2 vb0 = lds64(xa + offs[4 * i2 + 2]);
+        const uint2 vb1 = lds64(xa + offs[4 * i2 + 3]);
         const float2 wa0 = make_float2(w.x, w.x), wa1 = make_float2(w.y, w.y);
         const float2 wb0 = make_float2(w.z, w.z), wb1 = make_float2(w.w, w.w);
         a0 = __ffma2_rn(wa0, unpack2(va0.x), a0);
         a1 = __ffma2_rn(wa0, unpack2(va0.y), a1);
-        a2 = __ffma2_rn(wa0, unpack2(va0.z), a2);
-        a3 = __ffma2_rn(wa0, unpack2(va0.w), a3);
         b0 = __ffma2_rn(wb0, unpack2(vb0.x), b0);
         b1 = __ffma2_rn(wb0, unpack2(vb0.y), b1);
-        b2 = __ffma2_rn(wb0, unpack2(vb0.z), b2);
-        b3 = __ffma2_rn(wb0, unpack2(vb0.w), b3);
         a0 = __ffma2_rn(wa1, unpack2(va1.x), a0);
         a1 = __ffma2_rn(wa1, unpack2(va1.y), a1);
-        a2 = __ffma2_rn(wa1, unpack2(va1.z), a2);
-        a3 = __ffma2_rn(wa1, unpack2(va1.w), a3);
         b0 = __ffma2_rn(wb1, unpack2(vb1.x), b0);
         b1 = __ffma2_rn(wb1, unpack2(vb1.y), b1);
-        b2 = __ffma2_rn(wb1, unpack2(vb1.z), b2);
-        b3 = __ffma2_rn(wb1, unpack2(vb1.w), b3);
     }
 }
 
@@ -623,79 +714,68 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
     const uint32_t lx = (uint32_t)lig << 4;
     const int R = P.R, E = R + 1, kp = P.kp, NP = (R + 1) >> 1, Es = P.Es;
     const float *res = reinterpret_cast<const float *>(sm + P.off_res);
-    // this group's expert pair (warp w's groups take pairs w + 8h) and its
-    // row offsets, fixed for the whole launch; padding positions and the twin
-    // of an odd last expert read the zero row (their weights are 0)
-    const int pr = warp + kMixWarps * h;
+    // this group's expert pair (warps w and w + 8 take pairs (w mod 8) + 8h)
+    // and half hf of each 16-byte chunk (positions lig + 32 hf + 8 m, m < 4):
+    // the groups of a warp alternate halves, so a warp's 8-byte reads of four
+    // rows hit every bank twice; row offsets are fixed for the whole launch;
+    // padding positions and the twin of an odd last expert read the zero row
+    // (their weights are 0)
+    const int pr = (warp & (kPairWarps - 1)) + kPairWarps * h;
+    const int hf = (h & 1) ^ (warp / kPairWarps);
     const int ea = 2 * pr, eb = ea + 1;
     const bool pair_on = pr < NP;
-    uint32_t offs[kGateMaxK];
+    uint32_t offs[2 * kGateMaxK];
 #pragma unroll
     for (int i = 0; i < kGateMaxK; i += 2) {
-        uint32_t o[4];
 #pragma unroll
         for (int m = 0; m < 4; ++m) {
             const int e = m < 2 ? ea : eb, pos = i + (m & 1);
             const uint32_t c = (pair_on && e < R && pos < P.k)
                                    ? (uint32_t)__ldg(P.pidx + (size_t)e * P.k + pos)
                                    : (uint32_t)P.C;
-            o[m] = row_off(c, lx);
+            offs[2 * i + m] = row_off(c, lx) | ((uint32_t)hf << 3);
         }
-        offs[i] = o[0] | (o[1] << 16);
-        offs[i + 1] = o[2] | (o[3] << 16);
     }
-    uint32_t r = 0;
-    for (uint32_t it = blockIdx.x; it < P.items; it += gridDim.x, ++r) {
-        const uint32_t s = r % (uint32_t)P.D, tb = r % kNT, yb = r % kYB, rc = r % kRS;
-        const int n = (int)(it / (uint32_t)P.T), t = (int)(it - (uint32_t)n * P.T);
-        // one thread waits for the slot and the table, the others at the
-        // barrier; thread 0 has also seen the bulk copy of item r - kYB
-        // finish reading ys
+    const uint32_t sm_a = smem_u32(sm);
+    const uint32_t wlane = 16u * (uint32_t)(4 * (pr & 7) + (pr >> 3));  // wslot(pr, 0) * 16
+    for (Round q(P); q.live(P); q.next(P)) {
+        const uint32_t r = q.r, it = q.it, s = q.s;
+        const uint32_t tb = r % kNT, yb = r % kYB, rc = r % kRS;
+        const int n = q.n, t = q.t;
+        // three threads wait for the slot, the table and the residual column
+        // at once, the others at the barrier; thread 0 has also seen the bulk
+        // copy of item r - kYB finish reading ys
         bool ok = true;
-        if (st == 0) {
-            ok = ring_wait(mbar(P, sm, kMbFull + s), (r / P.D) & 1u, P.ctrl, it) &&
-                 ring_wait(mbar(P, sm, kMbTReady + tb), (r / kNT) & 1u, P.ctrl, it) &&
-                 ring_wait(mbar(P, sm, kMbRDone + rc), (r / kRS) & 1u, P.ctrl, it);
-        }
+        if (st == 0) ok = ring_wait(mbar(P, sm, kMbFull + s), q.ph, P.ctrl, it);
+        else if (st == 32) ok = ring_wait(mbar(P, sm, kMbTReady + tb), (r / kNT) & 1u, P.ctrl, it);
+        else if (st == 64) ok = ring_wait(mbar(P, sm, kMbRDone + rc), (r / kRS) & 1u, P.ctrl, it);
         if (!bar_and(kBarMix, kMixT, ok)) break;
-        const unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
         uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[yb]);
-        const float4 *wt = reinterpret_cast<const float4 *>(sm + P.off_tab[tb]);
         if (pair_on) {
-            float2 a0 = make_float2(0.f, 0.f), a1 = a0, a2 = a0, a3 = a0;
-            float2 b0 = a0, b1 = a0, b2 = a0, b3 = a0;
-            mix_pair_regs(xs, wt, pr, kp >> 1, offs, a0, a1, a2, a3, b0, b1, b2, b3);
-            // lane lig's positions are lig + 8 m
-            if (P.bulk_y) {
-                // rows of odd length: 16-bit stores
-                uint16_t *yh = ys + lig * Es + ea;
-                const int stp = kGS * Es;
-                const float av[8] = {a0.x, a0.y, a1.x, a1.y, a2.x, a2.y, a3.x, a3.y};
-                const float bv[8] = {b0.x, b0.y, b1.x, b1.y, b2.x, b2.y, b3.x, b3.y};
+            float2 a0 = make_float2(0.f, 0.f), a1 = a0, b0 = a0, b1 = a0;
+            mix_pair_half(sm_a + P.off_xs + s * P.xs_bytes, sm_a + P.off_tab[tb] + wlane, kp >> 1,
+                          offs, a0, a1, b0, b1);
+            // lane lig's positions are lig + 32 hf + 8 m
+            uint16_t *yh = ys + (lig + 32 * hf) * Es + ea;
+            const int stp = kGS * Es;
+            if (P.bulk_y || eb == R) {
+                // rows of odd length (or, for odd R, the twin's column is the
+                // residual column, written below by another thread): 16-bit
+                // stores
+                const float av[4] = {a0.x, a0.y, a1.x, a1.y};
+                const float bv[4] = {b0.x, b0.y, b1.x, b1.y};
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
+                for (int q = 0; q < 4; ++q) {
                     yh[q * stp] = f32_to_bf16(av[q]);
                     if (eb < R) yh[q * stp + 1] = f32_to_bf16(bv[q]);
                 }
-            } else if (eb == R) {
-                // odd R: the twin's column is the residual column, written
-                // below by another thread
-                uint16_t *yh = ys + lig * Es + ea;
-                const int stp = kGS * Es;
-                const float av[8] = {a0.x, a0.y, a1.x, a1.y, a2.x, a2.y, a3.x, a3.y};
-#pragma unroll
-                for (int q = 0; q < 8; ++q) yh[q * stp] = f32_to_bf16(av[q]);
             } else {
-                uint32_t *yw = reinterpret_cast<uint32_t *>(ys + lig * Es + ea);
-                const int stp = (kGS * Es) >> 1;
-                yw[0 * stp] = pack_bf16x2(a0.x, b0.x);
-                yw[1 * stp] = pack_bf16x2(a0.y, b0.y);
-                yw[2 * stp] = pack_bf16x2(a1.x, b1.x);
-                yw[3 * stp] = pack_bf16x2(a1.y, b1.y);
-                yw[4 * stp] = pack_bf16x2(a2.x, b2.x);
-                yw[5 * stp] = pack_bf16x2(a2.y, b2.y);
-                yw[6 * stp] = pack_bf16x2(a3.x, b3.x);
-                yw[7 * stp] = pack_bf16x2(a3.y, b3.y);
+                uint32_t *yw = reinterpret_cast<uint32_t *>(yh);
+                const int sw = stp >> 1;
+                yw[0 * sw] = pack_bf16x2(a0.x, b0.x);
+                yw[1 * sw] = pack_bf16x2(a0.y, b0.y);
+                yw[2 * sw] = pack_bf16x2(a1.x, b1.x);
+                yw[3 * sw] = pack_bf16x2(a1.y, b1.y);
             }
         }
         // the residual column (table role)
@@ -767,14 +847,6 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
     const uint32_t epoch = ld_relaxed(P.ctrl + kCtrlEpoch);
     const uint32_t tag = epoch + 1u;
     const bool loader = tid >= kLoad0 && tid < kTab0;
-    // the load role's first two tiles are in flight during the set-up
-    LoadUnits lu;
-    uint4 va[4], vb[4];
-    if (loader) {
-        lu = load_units(P, tid - kLoad0);
-        tile_loads(P, lu, blockIdx.x, va);
-        tile_loads(P, lu, blockIdx.x + gridDim.x, vb);
-    }
     // set-up: U list, the zero row of every slot, mbarriers
     int32_t *s_resid = reinterpret_cast<int32_t *>(sm + P.off_U);
     for (int i = tid; i < P.nU; i += kRingT) s_resid[i] = __ldg(P.resid + i);
@@ -784,6 +856,7 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
     }
     if (tid == 0) {
         for (int d = 0; d < P.D; ++d) {
+            mbar_init(mbar(P, sm, kMbRaw + d), 1);
             mbar_init(mbar(P, sm, kMbFull + d), 1);
             mbar_init(mbar(P, sm, kMbEmpty + d), 2);
         }
@@ -800,8 +873,9 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
     __syncthreads();
 
     if (tid < kMixT) mix_role(P, sm);
-    else if (loader) load_role(P, sm, lu, va, vb);
-    else table_role(P, sm, tag);
+    else if (loader) load_role(P, sm, load_units(P, tid - kLoad0));
+    else if (tid < kProd0) table_role(P, sm, tag);
+    else copy_role(P, sm);
 
     // the last CTA advances the epoch (the tag of the next forward)
     __syncthreads();
@@ -975,6 +1049,8 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
                                     (int)plan.smem)) != cudaSuccess)
         return err;
     const unsigned g2 = (unsigned)std::min<unsigned long long>(items, (unsigned long long)G);
+    P.Gn = (int)(g2 / (unsigned)T);
+    P.Gt = (int)(g2 % (unsigned)T);
     moce_ring_kernel<<<g2, kRingT, plan.smem, s>>>(P);
     return cudaGetLastError();
 }
