@@ -71,13 +71,18 @@ typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
  *                       C_in % 8 == 0, k <= 16, shared memory permitting)
  *   MOCE_PATH_STEPS     one kernel per step: pool, gate, mix (any layout
  *                       and dtype)
+ *   MOCE_PATH_RING      one cooperative kernel in which every CTA pools its
+ *                       tiles a few rounds before it mixes them, the CTA
+ *                       that pools an example's last tile runs the gate, and
+ *                       the second read of x comes from L2 (as TWO_PASS)
  */
 typedef enum moce_path {
     MOCE_PATH_AUTO = 0,
     MOCE_PATH_PIPE = 1,
     MOCE_PATH_TWO_PASS = 2,
     MOCE_PATH_FUSED = 3,
-    MOCE_PATH_STEPS = 4
+    MOCE_PATH_STEPS = 4,
+    MOCE_PATH_RING = 5
 } moce_path_t;
 
 /* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */

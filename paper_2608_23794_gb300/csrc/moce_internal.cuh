@@ -160,8 +160,8 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
                         const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
                         const float *W1, const float *b1, const float *w2, const float *b2,
                         float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
-                        cudaStream_t s);
+                        bool fused, cudaStream_t s);
 
-bool ring_supported(int N, int HW, int C, int R, int k);
+bool ring_supported(int N, int HW, int C, int R, int k, bool fused);
 
 }  // namespace moce

@@ -23,20 +23,21 @@
 // four lane groups of a mixing warp (pairs 8 apart) read different banks.
 //
 // Pass 2, moce_ring_kernel, reads x again and mixes it: one CTA per SM takes
-// items b, b + G, ...; its copy warp (19) brings each tile (64 positions x C
+// items b, b + G, ...; its copy warp (27) brings each tile (64 positions x C
 // channels, contiguous in NHWC) into a ring of D shared-memory slots by one
 // bulk copy as soon as a slot is free, so several tiles are in flight; the
-// load warps (8-15) transpose a landed tile in place to channel-major rows;
-// the table warps (16-18) bring the weights of the item two ahead into one of
-// four mixing tables by a bulk copy and sum the tile's unselected channels
-// for the residual expert (Eq. (res)); the mix warps (0-7) mix a slot with
-// its table: each group of 8 lanes owns 8 positions per lane and one expert
-// pair for the whole launch, whose row offsets it keeps in registers
-// (Eq. (expert)); the tile of y, residual column included, leaves by one bulk
-// copy. The roles hand slots and tables over through shared-memory
-// mbarriers; every wait is bounded and none crosses CTAs. No role holds
-// global loads in registers across a barrier: x and the weights arrive by
-// bulk copies, so the barriers never wait for HBM.
+// load warps (16-23) transpose a landed tile in place to channel-major rows;
+// the table warps (24-26) bring the weights of the item two ahead into one of
+// six mixing tables by a bulk copy and sum the tile's unselected channels for
+// the residual expert (Eq. (res)); the mix warps (0-15) mix two items per
+// round, each slot with its table: each group of 8 lanes owns one expert pair
+// and half of every 16-byte row chunk (4 positions per lane) for the whole
+// launch, with the pair's row offsets in registers (Eq. (expert)); each tile
+// of y, residual column included, leaves by one bulk copy. The roles hand
+// slots and tables over through shared-memory mbarriers; every wait is
+// bounded and none crosses CTAs. No role holds global loads in registers
+// across a barrier: x and the weights arrive by bulk copies, so the barriers
+// never wait for HBM.
 #include <algorithm>
 
 #include "moce_device.cuh"
@@ -60,10 +61,15 @@ constexpr int kTab0 = kMixT + kLoadT;            // first table thread
 constexpr int kProd0 = kTab0 + kTabT;            // the copy warp's first thread
 constexpr int kResParts = kTabT / 8;             // residual: U entries split kResParts ways
 constexpr int kPairWarps = 8;         // mix warps w and w + 8 share expert pairs
-constexpr int kNT = 4;                // mixing tables (weights arrive two items ahead)
-constexpr int kYB = 2;                // output tile buffers
+// Mixing tables: the weights of item r + 2 go into table (r + 2) mod kNT as
+// the table role starts item r, which must then wait only for items the mix
+// role has finished (r - 3 and before: a mixing round takes two items), so
+// kNT >= 2 + 3.
+constexpr int kNT = 6;
+constexpr int kYB = 4;                // output tile buffers (two items per mixing round)
 constexpr int kRS = 4;                // residual columns (the table role runs ahead)
 constexpr int kMaxD = 6;              // x slots at most
+constexpr int kLead = 10;             // single pass: rounds a CTA pools ahead of mixing
 constexpr int kGateMaxK = 16;          // support positions a mixing lane keeps in registers
 constexpr int kMaxPairs = 32;          // expert pairs: one per mixing group
 constexpr int kWBlock = kMaxPairs * 8; // float4 entries of a weight block
@@ -83,16 +89,18 @@ static_assert(kMixT == 2 * kPairWarps * 32, "two mix warps per set of expert pai
 static_assert(kTP == 8 * kGS, "a group's lanes cover the tile");
 static_assert(kPoolT == 4 * kTP, "pass 1: 32 channel blocks x 8 rows of positions");
 
-// Accumulator word of one (example, channel, group): bits 48-55 count the
-// runs published as fp32 instead, bits 0-47 hold the sum of
-// kFixBias + round(s * 2^20) over the fixed-point runs (s = the run's
-// channel sum, |s| < 2^19, so every term is in (0, 2^40) and any count of
-// runs below 256 fits).
+// Accumulator word of one (example, channel, group): bits 56-63 count the
+// runs added so far, bits 48-55 the runs published as fp32 instead, bits
+// 0-47 hold the sum of kFixBias + round(s * 2^20) over the fixed-point runs
+// (s = the run's channel sum, |s| < 2^19, so every term is in (0, 2^40) and
+// any count of runs below 256 fits). The gate reads a word only once its run
+// count is complete, so the adders need no fence before they count.
 constexpr float kFixScale = 1048576.0f;  // 2^20
 constexpr float kFixInv = 1.0f / 1048576.0f;
 constexpr float kFixMax = 524288.0f;     // 2^19
 constexpr unsigned long long kFixBias = 1ull << 39;
 constexpr unsigned long long kWideOne = 1ull << 48;
+constexpr unsigned long long kRunOne = 1ull << 56;
 
 // mbarriers of pass 2 (8 bytes each): raw[s] (the bulk copy of a tile into
 // slot s has landed: copy warp's arrival + transaction bytes), full[s]
@@ -143,9 +151,12 @@ struct RingParams {
     int bulk_y;                   // output tiles leave by one bulk copy
     uint32_t off_xs, xs_bytes;
     uint32_t off_tab[kNT], off_ys[kYB];
-    uint32_t off_res, off_rred, off_U, off_bar;
+    uint32_t off_res, off_rred, off_U, off_offs, off_bar;
     float inv_nU;                 // 1 / |U| (0 when U is empty)
     float inv_E;
+    int lead;                     // single pass: rounds a CTA pools ahead of mixing
+    uint32_t off_pool;            // single pass: the load role's pooling scratch
+    PoolParams pool;              // single pass: pooling and gate parameters
 };
 
 __device__ __forceinline__ void red_add_u64(unsigned long long *p, unsigned long long v) {
@@ -189,10 +200,9 @@ struct SupTab {
 template <int K>
 __device__ __noinline__ void gate_experts(const PoolParams &P, const float *W1t, const float *b1p,
                                           const float *w2p, const float *zs, const SupTab &S,
-                                          float4 *wts, float *tau_out) {
+                                          float4 *wts, float *tau_out, int st) {
     constexpr int TPE = K / 4;             // threads per expert
     constexpr int EPP = kPoolT / TPE;      // experts per pass
-    const int st = threadIdx.x;
     const int q = st % TPE, el = st / TPE;
     const int k = P.k, kp = P.kp;
     const float b2 = w2p[K];
@@ -243,7 +253,6 @@ __device__ __noinline__ void gate_experts(const PoolParams &P, const float *W1t,
         if (act) {
             const float inv = 1.f / s;
             // positions 4q .. 4q+3 are entries 2q and 2q+1 (the odd-k pad gets 0)
-            // positions 4q .. 4q+3 are entries 2q and 2q+1 (the odd-k pad gets 0)
             float *wf = reinterpret_cast<float *>(wts);
             const int pr = e >> 1, half = 2 * (e & 1);
             if (4 * q < kp)
@@ -269,12 +278,14 @@ struct PoolSmem {
     uint32_t last;
 };
 
-// The example's gate, by its last pooling CTA: z from the accumulator words
+// The example's gate, by the kPoolT threads (tid = 0 .. kPoolT - 1, meeting at
+// bar()) of the CTA that counted its last run: z from the accumulator words
 // (and the tagged fp32 run sums, in run order), then every expert's
 // temperature and weights; the accumulators and the counter are cleared for
-// the next forward.
-__device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t tag) {
-    const int tid = threadIdx.x;
+// the next forward, and made[n] = tag is published after everything else.
+template <typename Bar>
+__device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t tag, int tid,
+                               Bar bar) {
     const unsigned long long T = (unsigned long long)P.RPE;  // runs of the example
     unsigned long long *za = P.zacc + (size_t)n * kAccG * P.C;
     for (int c = tid; c < P.C; c += kPoolT) {
@@ -283,7 +294,14 @@ __device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t
 #pragma unroll
         for (int g = 0; g < kAccG; ++g) {
             const unsigned long long Tg = (T - (unsigned long long)g + kAccG - 1) / kAccG;
-            const unsigned long long w = __ldcg(za + (size_t)g * P.C + c);
+            // every run of the group has landed in the word (bounded)
+            unsigned long long w = ld_relaxed64(za + (size_t)g * P.C + c);
+            for (uint32_t i = 0; (w >> 56) != Tg && i < kSpinLimit; ++i) {
+                if ((i & 15u) == 15u && ld_relaxed(P.ctrl + kCtrlError) != 0u) break;
+                __nanosleep(64);
+                w = ld_relaxed64(za + (size_t)g * P.C + c);
+            }
+            if ((w >> 56) != Tg) report_timeout(P.ctrl, (uint32_t)n);
             const unsigned long long wg = (w >> 48) & 0xffull;
             fx += (long long)(w & ((1ull << 48) - 1ull)) - (long long)((Tg - wg) * kFixBias);
             wide = wide || wg != 0ull;
@@ -315,7 +333,7 @@ __device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t
         S.w2[P.Kg] = __ldg(P.b2);
         P.count[n] = 0u;
     }
-    __syncthreads();
+    bar();
     SupTab sup;
     sup.idx = P.pidx;
     sup.lg = P.plog;
@@ -325,11 +343,15 @@ __device__ void finish_example(const PoolParams &P, PoolSmem &S, int n, uint32_t
     // entries no expert writes (padding positions, the twin of an odd last
     // expert) stay 0
     for (int q = tid; q < kWBlock; q += kPoolT) wts[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-    __syncthreads();
+    bar();
     float *tau = P.tau + (size_t)n * P.R;
-    if (P.Kg == 16) gate_experts<16>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau);
-    else gate_experts<32>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau);
-    if (tid == 0) P.made[n] = tag;  // read by pass 2 after this kernel ends
+    if (P.Kg == 16) gate_experts<16>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau, tid);
+    else gate_experts<32>(P, S.W1t, S.b1, S.w2, S.zs, sup, wts, tau, tid);
+    // the weights, z and tau are visible before the tag: mixing CTAs of the
+    // same launch read it with acquire
+    __threadfence();
+    bar();
+    if (tid == 0) st_release(P.made + n, tag);
 }
 
 // A CTA pools one run of up to RL consecutive tiles of one example: thread
@@ -379,11 +401,11 @@ __global__ void __launch_bounds__(kPoolT) moce_poolgate_kernel(const PoolParams 
             for (int q = 0; q < 8; ++q) s += S.red[q * P.C + tid];
             unsigned long long add;
             if (fabsf(s) < kFixMax) {
-                add = kFixBias + (unsigned long long)__float2ll_rn(s * kFixScale);
+                add = kRunOne + kFixBias + (unsigned long long)__float2ll_rn(s * kFixScale);
             } else {  // beyond the fixed-point range (or NaN): a tagged fp32 word
                 P.part[((size_t)n * P.RPE + j) * P.C + tid] =
                     ((unsigned long long)tag << 32) | __float_as_uint(s);
-                add = kWideOne;
+                add = kRunOne + kWideOne;
             }
             red_add_u64(P.zacc + ((size_t)n * kAccG + (j % kAccG)) * P.C + tid, add);
             __threadfence();
@@ -402,7 +424,7 @@ __global__ void __launch_bounds__(kPoolT) moce_poolgate_kernel(const PoolParams 
         }
         __syncthreads();
         if (S.last) {
-            finish_example(P, S, n, tag);
+            finish_example(P, S, n, tag, tid, [] { __syncthreads(); });
             __syncthreads();
         }
     }
@@ -444,25 +466,18 @@ __device__ __forceinline__ LoadUnits load_units(const RingParams &P, int lt) {
     return u;
 }
 
-// A role's position in its items b, b + G, ...: round r, item it (example n,
-// tile t), slot s = r mod D and its phase bit (r / D) mod 2, advanced
-// without divisions.
-struct Round {
-    uint32_t r, it, s, ph;
+// A CTA's items are b, b + G, ... (rounds r = 0 .. nb - 1); ItemPos follows
+// one of them (item it: example n, tile t) without divisions.
+struct ItemPos {
+    uint32_t r, it;
     int n, t;
-    __device__ __forceinline__ explicit Round(const RingParams &P)
-        : r(0), it(blockIdx.x), s(0), ph(0) {
+    __device__ __forceinline__ explicit ItemPos(const RingParams &P) : r(0), it(blockIdx.x) {
         n = (int)(blockIdx.x / (uint32_t)P.T);
         t = (int)blockIdx.x - n * P.T;
     }
-    __device__ __forceinline__ bool live(const RingParams &P) const { return it < P.items; }
     __device__ __forceinline__ void next(const RingParams &P) {
         ++r;
         it += gridDim.x;
-        if (++s == (uint32_t)P.D) {
-            s = 0;
-            ph ^= 1u;
-        }
         n += P.Gn;
         t += P.Gt;
         if (t >= P.T) {
@@ -474,39 +489,156 @@ struct Round {
     __device__ __forceinline__ int np(const RingParams &P) const { return min(kTP, P.HW - t * kTP); }
 };
 
-// The copy warp: one bulk copy per item of the tile's np * C contiguous bf16
-// (NHWC) into slot r mod D, once the mix and table roles have released the
-// slot; raw[s] completes when the bytes have landed. On a wait that gave up,
-// the copies still in flight land before the warp returns.
+// The CTA's slot sequence: every position j takes slot j mod D (phase bit
+// (j / D) mod 2 of the slot's raw and empty mbarriers) for one tile; full[s]
+// completes only for mixing positions, so the roles that wait on it keep one
+// phase bit per slot (FullPhase). A two-pass launch only
+// mixes: position r holds item r. A single-pass launch also pools its own
+// items L = lead rounds ahead: positions pool(0 .. L - 1), then per round r
+// pool(r + L) (while there is one) and mix(r). Every role walks the same
+// sequence. F: a single-pass launch.
+template <bool F>
+struct Seq {
+    ItemPos pool, mix;  // next pool item, next mix item
+    uint32_t j, s, ph;  // position, slot, phase bit
+    uint32_t nb;        // items of this CTA
+    bool is_pool;       // the position pools (else it mixes mix)
+    __device__ __forceinline__ explicit Seq(const RingParams &P)
+        : pool(P), mix(P), j(0), s(0), ph(0) {
+        nb = (P.items - blockIdx.x + gridDim.x - 1) / gridDim.x;
+        decide(P);
+    }
+    __device__ __forceinline__ void decide(const RingParams &P) {
+        is_pool = F && pool.r < nb && pool.r < mix.r + (uint32_t)P.lead;
+    }
+    __device__ __forceinline__ bool live() const { return mix.r < nb; }
+    __device__ __forceinline__ const ItemPos &item() const { return is_pool ? pool : mix; }
+    __device__ __forceinline__ void next(const RingParams &P) {
+        if (is_pool) pool.next(P);
+        else mix.next(P);
+        ++j;
+        if (++s == (uint32_t)P.D) {
+            s = 0;
+            ph ^= 1u;
+        }
+        decide(P);
+    }
+    // the next mixing position
+    __device__ __forceinline__ void next_mix(const RingParams &P) {
+        do next(P);
+        while (live() && is_pool);
+    }
+};
+
+// Example n's tag: with acquire in a single-pass launch (the gate ran in
+// another CTA of it), else relaxed (pass 1 has finished).
+template <bool F>
+__device__ __forceinline__ uint32_t read_tag(const RingParams &P, int n) {
+    return F ? ld_acquire(P.made + n) : ld_relaxed(P.made + n);
+}
+
+// Waits until example n's gate has run in this forward (made[n] == tag,
+// read with acquire; v is a value already read). A two-pass launch starts
+// after pass 1 has finished, so there a stale tag is reported at once; a
+// single-pass launch waits (bounded) for the CTA that pools the example's
+// last tile. False when the wait gave up or another wait did.
+template <bool F>
+__device__ bool made_wait(const RingParams &P, int n, uint32_t tag, uint32_t v, uint32_t it) {
+    for (uint32_t i = 1; v != tag; ++i) {
+        if (!F || i >= kSpinLimit) {
+            report_timeout(P.ctrl, it);
+            return false;
+        }
+        if ((i & 15u) == 0u && ld_relaxed(P.ctrl + kCtrlError) != 0u) return false;
+        __nanosleep(64);
+        v = read_tag<F>(P, n);
+    }
+    return true;
+}
+
+// Slot of mixing item m (round m of the CTA, nb items): its position is m
+// in a two-pass launch; in a single-pass launch with L = min(lead, nb) pooled
+// positions first it is L + 2 m while pooled positions still follow, then
+// nb + m.
+template <bool F>
+__device__ __forceinline__ uint32_t mix_slot(const RingParams &P, uint32_t m, uint32_t nb) {
+    uint32_t pos = m;
+    if (F) {
+        const uint32_t L = min((uint32_t)P.lead, nb);
+        pos = m < nb - L ? L + 2u * m : nb + m;
+    }
+    return pos % (uint32_t)P.D;
+}
+__device__ __forceinline__ uint32_t cta_items(const RingParams &P) {
+    return (P.items - blockIdx.x + gridDim.x - 1) / gridDim.x;
+}
+
+// Phase bits of the full mbarriers, one per slot: a role that waits for
+// every mixing use of every slot in order flips slot s's bit after each wait.
+struct FullPhase {
+    uint32_t bits = 0;
+    __device__ __forceinline__ uint32_t take(uint32_t s) {
+        const uint32_t b = (bits >> s) & 1u;
+        bits ^= 1u << s;
+        return b;
+    }
+};
+
+// One bulk copy of the weight block of mix item q's example into table
+// q.r mod kNT; tready of that table completes when the 4 KB have landed.
+__device__ __forceinline__ void weights_copy(const RingParams &P, unsigned char *sm,
+                                             const ItemPos &q) {
+    const uint32_t tb = q.r % kNT;
+    const uint32_t bar = mbar(P, sm, kMbTReady + tb);
+    // the weights were written by generic stores (of this launch, read
+    // with acquire, or of pass 1); the mix role's reads of the table's
+    // previous contents come first
+    asm volatile(
+        "fence.proxy.async.global;\n\t"
+        "fence.proxy.async.shared::cta;\n\t"
+        "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, "
+        "[%0];" ::"r"(bar),
+        "r"((uint32_t)(kWBlock * 16)), "r"(smem_u32(sm + P.off_tab[tb])),
+        "l"(P.wts + (size_t)q.n * kWBlock)
+        : "memory");
+}
+
+// The copy warp walks the slot sequence: per position, once the slot is
+// released (empty[s]: the mix and table roles, or the load role for a
+// pooled tile), one bulk copy of the tile's np * C contiguous bf16 (NHWC);
+// raw[s] completes when the bytes have landed. On a wait that gave up, the
+// copies still in flight land before the warp returns.
+template <bool F>
 __device__ void copy_role(const RingParams &P, unsigned char *sm) {
     set_role_regs<kTabRegs, kLaunchRegs>();
     if ((threadIdx.x & 31) == 0) {
-        Round q(P);
+        Seq<F> q(P);
         bool ok = true;
-        for (; q.live(P); q.next(P)) {
-            if (q.r >= (uint32_t)P.D &&
-                !ring_wait(mbar(P, sm, kMbEmpty + q.s), q.ph ^ 1u, P.ctrl, q.it)) {
+        for (; q.live(); q.next(P)) {
+            if (q.j >= (uint32_t)P.D &&
+                !ring_wait(mbar(P, sm, kMbEmpty + q.s), q.ph ^ 1u, P.ctrl, q.item().it)) {
                 ok = false;
                 break;
             }
-            const uint32_t bytes = (uint32_t)q.np(P) * (uint32_t)P.C * 2u;
-            const uint16_t *src = P.x + ((size_t)q.n * P.HW + q.p0()) * P.C;
-            const uint32_t s = q.s;
-            const uint32_t bar = mbar(P, sm, kMbRaw + s);
+            const ItemPos &w = q.item();
+            const uint32_t bytes = (uint32_t)w.np(P) * (uint32_t)P.C * 2u;
+            const uint16_t *src = P.x + ((size_t)w.n * P.HW + w.p0()) * P.C;
+            const uint32_t bar = mbar(P, sm, kMbRaw + q.s);
             // the slot's earlier generic-proxy reads and writes come before the copy
             asm volatile(
                 "fence.proxy.async.shared::cta;\n\t"
                 "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
                 "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, "
                 "[%0];" ::"r"(bar),
-                "r"(bytes), "r"(smem_u32(sm + P.off_xs + s * P.xs_bytes)), "l"(src)
+                "r"(bytes), "r"(smem_u32(sm + P.off_xs + q.s * P.xs_bytes)), "l"(src)
                 : "memory");
         }
         if (!ok) {
-            const uint32_t r = q.r;
-            for (uint32_t j = r > (uint32_t)P.D ? r - (uint32_t)P.D : 0u; j < r; ++j) {
-                const uint32_t bar = mbar(P, sm, kMbRaw + j % (uint32_t)P.D);
-                for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (j / P.D) & 1u); ++i)
+            const uint32_t j1 = q.j, d = (uint32_t)P.D;
+            for (uint32_t j = j1 > d ? j1 - d : 0u; j < j1; ++j) {
+                const uint32_t bar = mbar(P, sm, kMbRaw + j % d);
+                for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (j / d) & 1u); ++i)
                     __nanosleep(256);
             }
         }
@@ -514,22 +646,123 @@ __device__ void copy_role(const RingParams &P, unsigned char *sm) {
     __syncwarp();
 }
 
-// The load role, per item r: once raw[s] completes, every thread reads its
-// staging units of the raw tile in slot s (positions past np read as 0),
-// the role meets at a barrier, and the units are written back in place as
-// channel-major rows of pixel pairs (the raw tile, np * C * 2 bytes, lies
-// within rows 0 .. C - 1, so row C stays zero).
-__device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnits &u) {
+// A pooled position (single-pass launches), by the load role: thread
+// (row = lt / 32, cb = lt mod 32) adds positions row, row + 8, ... of
+// channels 8 cb .. 8 cb + 7 of the raw tile, the eight rows are added in
+// order through shared memory, the slot is released, and thread c adds the
+// tile's channel sum c to the example's accumulator words (group t mod kAccG)
+// as in pass 1 (run count included). After the role's barrier thread 0
+// counts the tile; the count it gets back is looked at two positions later
+// (gate_if_last), so the role does not wait for it.
+__device__ __forceinline__ void pool_tile(const RingParams &P, unsigned char *sm,
+                                          const unsigned char *xs, const ItemPos &w, uint32_t s,
+                                          uint32_t tag, uint32_t drop, uint32_t &old) {
+    const int lt = threadIdx.x - kLoad0;
+    const int row = lt >> 5, cb = lt & 31;
+    PoolSmem &S = *reinterpret_cast<PoolSmem *>(sm + P.off_pool);
+    const int np = w.np(P);
+    float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (8 * cb < P.C) {
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const int p = row + 8 * m;
+            if (p < np) {
+                const uint4 v = lds128(xs + 2 * (p * P.C + 8 * cb));
+                a[0] += bf16lo(v.x); a[1] += bf16hi(v.x);
+                a[2] += bf16lo(v.y); a[3] += bf16hi(v.y);
+                a[4] += bf16lo(v.z); a[5] += bf16hi(v.z);
+                a[6] += bf16lo(v.w); a[7] += bf16hi(v.w);
+            }
+        }
+        float4 *rr = reinterpret_cast<float4 *>(S.red + row * P.C + 8 * cb);
+        rr[0] = make_float4(a[0], a[1], a[2], a[3]);
+        rr[1] = make_float4(a[4], a[5], a[6], a[7]);
+    }
+    bar_sync(kBarLoad, kLoadT);  // the raw tile is read; the row sums are complete
+    if (lt == 0) {
+        // the slot is free (two arrivals, as the mix and table roles give it)
+        mbar_arrive(mbar(P, sm, kMbEmpty + s));
+        mbar_arrive(mbar(P, sm, kMbEmpty + s));
+    }
+    const PoolParams &Q = P.pool;
+    const bool counted = w.it + 1u != drop;  // fault injection: this tile is never counted
+    if (lt < P.C && counted) {
+        float sum = 0.f;
+#pragma unroll
+        for (int qq = 0; qq < 8; ++qq) sum += S.red[qq * P.C + lt];
+        unsigned long long add;
+        if (fabsf(sum) < kFixMax) {
+            add = kRunOne + kFixBias + (unsigned long long)__float2ll_rn(sum * kFixScale);
+        } else {  // beyond the fixed-point range (or NaN): a tagged fp32 word
+            Q.part[((size_t)w.n * P.T + w.t) * P.C + lt] =
+                ((unsigned long long)tag << 32) | __float_as_uint(sum);
+            __threadfence();  // the word is visible before the run is counted in it
+            add = kRunOne + kWideOne;
+        }
+        red_add_u64(Q.zacc + ((size_t)w.n * kAccG + (w.t % kAccG)) * P.C + lt, add);
+    }
+    bar_sync(kBarLoad, kLoadT);  // every channel of the tile is added; red is free again
+    if (lt == 0 && counted) old = atomicAdd(Q.count + w.n, 1u);
+}
+
+// The count of a pooled tile (thread 0's old), looked at one position later:
+// the CTA that counted the example's last tile runs its gate with the load
+// role's threads.
+__device__ __forceinline__ void gate_if_last(const RingParams &P, unsigned char *sm, int n,
+                                             uint32_t old, uint32_t tag) {
+    const int lt = threadIdx.x - kLoad0;
+    PoolSmem &S = *reinterpret_cast<PoolSmem *>(sm + P.off_pool);
+    if (lt == 0) {
+        const uint32_t last = old == (uint32_t)P.T - 1u ? 1u : 0u;
+        S.last = last;
+    }
+    bar_sync(kBarLoad, kLoadT);
+    if (S.last) {
+        finish_example(P.pool, S, n, tag, lt, [] { bar_sync(kBarLoad, kLoadT); });
+        bar_sync(kBarLoad, kLoadT);
+    }
+}
+
+// The load role walks the slot sequence: once raw[s] completes, a pooled
+// position is reduced (pool_tile); a mixing position is read unit by unit
+// (positions past np read as 0), the role meets at a barrier, and the units
+// are written back in place as channel-major rows of pixel pairs (the raw
+// tile, np * C * 2 bytes, lies within rows 0 .. C - 1, so row C stays zero);
+// full[s] then tells the mix and table roles.
+template <bool F>
+__device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnits &u,
+                          uint32_t tag) {
     set_role_regs<kLoadRegs, kLaunchRegs>();
     const int lt = threadIdx.x - kLoad0;
     const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
-    for (Round q(P); q.live(P); q.next(P)) {
+    const uint32_t drop = ld_relaxed(P.ctrl + kCtrlDropItem);
+    // the last two pooled tiles whose counts have not been looked at:
+    // example (-1: none) and, in thread 0, the count it got back
+    int pend0 = -1, pend1 = -1;
+    uint32_t old0 = 0xffffffffu, old1 = 0xffffffffu;
+    Seq<F> q(P);
+    for (; q.live(); q.next(P)) {
         const uint32_t s = q.s;
         bool ok = true;
-        if (lt == 0) ok = ring_wait(mbar(P, sm, kMbRaw + s), q.ph, P.ctrl, q.it);
+        if (lt == 0) ok = ring_wait(mbar(P, sm, kMbRaw + s), q.ph, P.ctrl, q.item().it);
         if (!bar_and(kBarLoad, kLoadT, ok)) return;
-        const int np = q.np(P);
+        // the older pending count is looked at every position (the last
+        // pooled tiles' gates must not wait for the end of the sequence:
+        // mixing positions after them may need those examples)
         unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
+        if constexpr (F) {
+            if (pend0 >= 0) gate_if_last(P, sm, pend0, old0, tag);
+            pend0 = pend1;
+            old0 = old1;
+            pend1 = -1;
+            if (q.is_pool) {
+                old1 = 0xffffffffu;
+                pool_tile(P, sm, xs, q.pool, s, tag, drop, old1);
+                pend1 = q.pool.n;
+                continue;
+            }
+        }
+        const int np = q.mix.np(P);
         uint4 v[2 * kLU];
 #pragma unroll
         for (int i = 0; i < kLU; ++i) {
@@ -555,32 +788,20 @@ __device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnit
         bar_sync(kBarLoad, kLoadT);
         if (lt == 0) mbar_arrive(mbar(P, sm, kMbFull + s));
     }
+    if constexpr (F) {
+        if (pend0 >= 0) gate_if_last(P, sm, pend0, old0, tag);
+        if (pend1 >= 0) gate_if_last(P, sm, pend1, old1, tag);
+    }
 }
 
-// The table role, per item r: copies the weights of the item's example
-// (pass 1) into table r mod kNT (an example whose weights pass 1 of this
-// forward did not produce, because a tile was never counted, is reported as
-// MOCE_ERR_TIMEOUT); then, once the tile is staged, the residual expert
-// (Eq. (res)): thread (q = chunk, part) adds U entries part, part +
-// kResParts, ... for the chunk's 8 positions, the parts are added in order,
-// and res[r mod kYB][p] = sum / |U| (0 if U is empty).
-// One bulk copy of the weight block of round q's example into table
-// q.r mod kNT; tready of that table completes when the 4 KB have landed.
-__device__ __forceinline__ void weights_copy(const RingParams &P, unsigned char *sm,
-                                             const Round &q) {
-    const uint32_t tb = q.r % kNT;
-    const uint32_t bar = mbar(P, sm, kMbTReady + tb);
-    // the mix role's reads of the table's previous contents come first
-    asm volatile(
-        "fence.proxy.async.shared::cta;\n\t"
-        "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t"
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%2], [%3], %1, "
-        "[%0];" ::"r"(bar),
-        "r"((uint32_t)(kWBlock * 16)), "r"(smem_u32(sm + P.off_tab[tb])),
-        "l"(P.wts + (size_t)q.n * kWBlock)
-        : "memory");
-}
-
+// The table role walks the mixing positions. Its thread 0 brings the weights
+// of the item two ahead: once table (r + 2) mod kNT is released (the mix role
+// finished item r + 2 - kNT) and the example's gate has run in this forward
+// (made_wait), one bulk copy into the table. Then, once the tile is staged,
+// the residual expert (Eq. (res)): thread (q = chunk, part) adds U entries
+// part, part + kResParts, ... for the chunk's 8 positions, the parts are added
+// in order, and res[r mod kRS][p] = sum / |U| (0 if U is empty).
+template <bool F>
 __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag) {
     set_role_regs<kTabRegs, kLaunchRegs>();
     const int tt = threadIdx.x - kTab0;
@@ -588,34 +809,33 @@ __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag)
     const uint32_t lx = (uint32_t)q << 4;
     const int32_t *s_resid = reinterpret_cast<const int32_t *>(sm + P.off_U);
     float *rred = reinterpret_cast<float *>(sm + P.off_rred);
-    // thread 0 keeps the weights of the next two items in flight
-    Round ahead(P);
+    const uint32_t nb = cta_items(P);
+    FullPhase fph;
+    // thread 0: the next item whose weights to bring, and the copies made
+    ItemPos wq(P);
+    uint32_t wcopies = 0;
+    bool wok = true;
     if (tt == 0) {
-        for (int i = 0; i < 2 && ahead.live(P); ++i) {
-            weights_copy(P, sm, ahead);
-            ahead.next(P);
+        for (int i = 0; i < 2 && wok && wq.r < nb; ++i) {
+            wok = made_wait<F>(P, wq.n, tag, read_tag<F>(P, wq.n), wq.it);
+            if (wok) weights_copy(P, sm, wq), ++wcopies, wq.next(P);
         }
     }
-    for (Round rd(P); rd.live(P); rd.next(P)) {
-        const uint32_t r = rd.r, it = rd.it, s = rd.s;
+    for (ItemPos mi(P); mi.r < nb; mi.next(P)) {
+        const uint32_t r = mi.r, it = mi.it, s = mix_slot<F>(P, r, nb);
         const uint32_t rc = r % kRS;
-        const int n = rd.n;
-        bool ok = true;
+        const uint32_t fp = fph.take(s);
+        bool ok = wok;
+        if (tt == 0 && ok && wq.r < nb) {
+            const uint32_t tb = wq.r % kNT;
+            if (wq.r >= (uint32_t)kNT)
+                ok = ring_wait(mbar(P, sm, kMbTFree + tb), ((wq.r / kNT) - 1u) & 1u, P.ctrl, it);
+            if (ok) ok = made_wait<F>(P, wq.n, tag, read_tag<F>(P, wq.n), wq.it);
+            if (ok) weights_copy(P, sm, wq), ++wcopies, wq.next(P);
+            wok = ok;
+        }
         if (tt == 0) {
-            if (__ldg(P.made + n) != tag) report_timeout(P.ctrl, it);
-            if (ahead.live(P)) {
-                // table ahead.r mod kNT is free once the mix role is done with
-                // item ahead.r - kNT
-                const uint32_t tb = ahead.r % kNT;
-                if (ahead.r >= (uint32_t)kNT)
-                    ok = ring_wait(mbar(P, sm, kMbTFree + tb), ((ahead.r / kNT) - 1u) & 1u,
-                                   P.ctrl, it);
-                if (ok) {
-                    weights_copy(P, sm, ahead);
-                    ahead.next(P);
-                }
-            }
-            if (ok) ok = ring_wait(mbar(P, sm, kMbFull + s), rd.ph, P.ctrl, it);
+            if (ok) ok = ring_wait(mbar(P, sm, kMbFull + s), fp, P.ctrl, it);
             if (ok && r >= (uint32_t)kRS)
                 ok = ring_wait(mbar(P, sm, kMbRFree + rc), ((r / kRS) - 1u) & 1u, P.ctrl, it);
         }
@@ -645,13 +865,12 @@ __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag)
         bar_sync(kBarTab, kTabT);  // rred is free again; the residual column is complete
         if (tt == 0) mbar_arrive(mbar(P, sm, kMbRDone + rc));
     }
-    // after a wait gave up, the weight copies still in flight land before the
+    // after a wait gave up, weight copies still in flight land before the
     // CTA exits (after a normal end the mix role has waited for all of them)
-    if (tt == 0 && ahead.r > 0) {
-        const uint32_t last = ahead.r;
-        for (uint32_t j = last > (uint32_t)kNT ? last - (uint32_t)kNT : 0u; j < last; ++j) {
-            const uint32_t bar = mbar(P, sm, kMbTReady + j % kNT);
-            for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (j / kNT) & 1u); ++i)
+    if (tt == 0) {
+        for (uint32_t m = wcopies > (uint32_t)kNT ? wcopies - (uint32_t)kNT : 0u; m < wcopies; ++m) {
+            const uint32_t bar = mbar(P, sm, kMbTReady + m % kNT);
+            for (uint32_t i = 0; i < kSpinLimit && !mbar_test(bar, (m / kNT) & 1u); ++i)
                 __nanosleep(256);
         }
     }
@@ -678,34 +897,65 @@ __device__ __forceinline__ float4 lds128f(uint32_t a) {
     return v;
 }
 
-// Weighted sums of the lane's expert pair for its 4 positions: per entry i2,
-// one float4 of weights (at wa + 512 i2) and four 8-byte halves of row
-// chunks at xa + offs[4 i2 + j] (j = 0, 1: expert a, support positions 2 i2,
-// 2 i2 + 1; j = 2, 3: expert b).
-__device__ __forceinline__ void mix_pair_half(uint32_t xa, uint32_t wa, int npairs,
-                                              const uint32_t *offs, float2 &a0, float2 &a1,
+// bf16 pair -> two fp32: the low half by an integer multiply (FMA pipe),
+// the high half by a mask (ALU pipe), so the two pipes share the unpacking.
+__device__ __forceinline__ float2 unpack2_split(uint32_t w) {
+    uint32_t lo;
+    asm("mul.lo.u32 %0, %1, 65536;" : "=r"(lo) : "r"(w));
+    return make_float2(__uint_as_float(lo), __uint_as_float(w & 0xffff0000u));
+}
+
+// Weighted sums of the lane's expert pair for its 4 positions. Entry i2 of
+// the pair is one float4 of weights (at wa + 512 i2) and four 8-byte halves
+// of row chunks at xa + the 16-bit offsets of the pair's offset word
+// (at oa + 256 i2: {expert a, expert b}, support positions 2 i2 and 2 i2 + 1
+// in the low and high half, XORed with the lane's chunk and half, lxx).
+// Entry i2 + 1's reads are issued before entry i2 is added and the offsets
+// two entries ahead, so a lane keeps shared-memory reads in flight while it
+// computes.
+struct MixEntry {
+    float4 w;
+    uint2 a0, a1, b0, b1;
+};
+__device__ __forceinline__ MixEntry mix_load(uint32_t xa, uint32_t wa, uint2 o, uint32_t lxx,
+                                             int i2) {
+    MixEntry m;
+    const uint32_t oa = o.x ^ lxx, ob = o.y ^ lxx;
+    m.w = lds128f(wa + 512u * i2);
+    m.a0 = lds64(xa + (oa & 0xffffu));
+    m.a1 = lds64(xa + (oa >> 16));
+    m.b0 = lds64(xa + (ob & 0xffffu));
+    m.b1 = lds64(xa + (ob >> 16));
+    return m;
+}
+__device__ __forceinline__ void mix_pair_half(uint32_t xa, uint32_t wa, uint32_t oa,
+                                              uint32_t lxx, int npairs, float2 &a0, float2 &a1,
                                               float2 &b0, float2 &b1) {
+    uint2 on = lds64(oa + 256u);
+    MixEntry cur = mix_load(xa, wa, lds64(oa), lxx, 0);
 #pragma unroll
     for (int i2 = 0; i2 < kGateMaxK / 2; ++i2) {
         if (i2 >= npairs) break;
-        const float4 w = lds128f(wa + 512u * i2);
-        const uint2 va0 = lds64(xa + offs[4 * i2 + 0]);
-        const uint2 va1 = lds64(xa + offs[4 * i2 + 1]);
-        const uint2 vb0 = lds64(xa + offs[4 * i2 + 2]);
-        const uint2 vb1 = lds64(xa + offs[4 * i2 + 3]);
-        const float2 wa0 = make_float2(w.x, w.x), wa1 = make_float2(w.y, w.y);
-        const float2 wb0 = make_float2(w.z, w.z), wb1 = make_float2(w.w, w.w);
-        a0 = __ffma2_rn(wa0, unpack2(va0.x), a0);
-        a1 = __ffma2_rn(wa0, unpack2(va0.y), a1);
-        b0 = __ffma2_rn(wb0, unpack2(vb0.x), b0);
-        b1 = __ffma2_rn(wb0, unpack2(vb0.y), b1);
-        a0 = __ffma2_rn(wa1, unpack2(va1.x), a0);
-        a1 = __ffma2_rn(wa1, unpack2(va1.y), a1);
-        b0 = __ffma2_rn(wb1, unpack2(vb1.x), b0);
-        b1 = __ffma2_rn(wb1, unpack2(vb1.y), b1);
+        MixEntry nxt = cur;
+        if (i2 + 1 < kGateMaxK / 2 && i2 + 1 < npairs) {
+            nxt = mix_load(xa, wa, on, lxx, i2 + 1);
+            if (i2 + 2 < kGateMaxK / 2 && i2 + 2 < npairs) on = lds64(oa + 256u * (i2 + 2));
+        }
+        const float2 wa0 = make_float2(cur.w.x, cur.w.x), wa1 = make_float2(cur.w.y, cur.w.y);
+        const float2 wb0 = make_float2(cur.w.z, cur.w.z), wb1 = make_float2(cur.w.w, cur.w.w);
+        a0 = __ffma2_rn(wa0, unpack2_split(cur.a0.x), a0);
+        a1 = __ffma2_rn(wa0, unpack2_split(cur.a0.y), a1);
+        b0 = __ffma2_rn(wb0, unpack2_split(cur.b0.x), b0);
+        b1 = __ffma2_rn(wb0, unpack2_split(cur.b0.y), b1);
+        a0 = __ffma2_rn(wa1, unpack2_split(cur.a1.x), a0);
+        a1 = __ffma2_rn(wa1, unpack2_split(cur.a1.y), a1);
+        b0 = __ffma2_rn(wb1, unpack2_split(cur.b1.x), b0);
+        b1 = __ffma2_rn(wb1, unpack2_split(cur.b1.y), b1);
+        cur = nxt;
     }
 }
 
+template <bool F>
 __device__ void mix_role(const RingParams &P, unsigned char *sm) {
     set_role_regs<kMixRegs, kLaunchRegs>();
     const int st = threadIdx.x;
@@ -724,37 +974,36 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
     const int hf = (h & 1) ^ (warp / kPairWarps);
     const int ea = 2 * pr, eb = ea + 1;
     const bool pair_on = pr < NP;
-    uint32_t offs[2 * kGateMaxK];
-#pragma unroll
-    for (int i = 0; i < kGateMaxK; i += 2) {
+    // the offset table: entry (pair p, i2) at wslot(p, i2), two words of
+    // row offsets without the lane's chunk (thread (p, i2) writes it)
+    const uint32_t sm_a = smem_u32(sm);
+    if (st < kWBlock) {
+        const int p = st >> 3, i2 = st & 7;
+        uint32_t o[4];
 #pragma unroll
         for (int m = 0; m < 4; ++m) {
-            const int e = m < 2 ? ea : eb, pos = i + (m & 1);
-            const uint32_t c = (pair_on && e < R && pos < P.k)
+            const int e = 2 * p + (m >> 1), pos = 2 * i2 + (m & 1);
+            const uint32_t c = (2 * p < R + 1 && e < R && pos < P.k)
                                    ? (uint32_t)__ldg(P.pidx + (size_t)e * P.k + pos)
                                    : (uint32_t)P.C;
-            offs[2 * i + m] = row_off(c, lx) | ((uint32_t)hf << 3);
+            o[m] = row_off(c, 0u);
         }
+        uint2 *ot = reinterpret_cast<uint2 *>(sm + P.off_offs);
+        ot[wslot(p, i2)] = make_uint2(o[0] | (o[1] << 16), o[2] | (o[3] << 16));
     }
-    const uint32_t sm_a = smem_u32(sm);
+    bar_sync(kBarMix, kMixT);
+    const uint32_t lxx = (lx | ((uint32_t)hf << 3)) * 0x10001u;
     const uint32_t wlane = 16u * (uint32_t)(4 * (pr & 7) + (pr >> 3));  // wslot(pr, 0) * 16
-    for (Round q(P); q.live(P); q.next(P)) {
-        const uint32_t r = q.r, it = q.it, s = q.s;
-        const uint32_t tb = r % kNT, yb = r % kYB, rc = r % kRS;
-        const int n = q.n, t = q.t;
-        // three threads wait for the slot, the table and the residual column
-        // at once, the others at the barrier; thread 0 has also seen the bulk
-        // copy of item r - kYB finish reading ys
-        bool ok = true;
-        if (st == 0) ok = ring_wait(mbar(P, sm, kMbFull + s), q.ph, P.ctrl, it);
-        else if (st == 32) ok = ring_wait(mbar(P, sm, kMbTReady + tb), (r / kNT) & 1u, P.ctrl, it);
-        else if (st == 64) ok = ring_wait(mbar(P, sm, kMbRDone + rc), (r / kRS) & 1u, P.ctrl, it);
-        if (!bar_and(kBarMix, kMixT, ok)) break;
-        uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[yb]);
+    const uint32_t olane = sm_a + P.off_offs + 8u * (uint32_t)(4 * (pr & 7) + (pr >> 3));
+    // item q: mix the slot with its table into ys[q.r mod kYB] and add the
+    // residual column
+    auto mix_item = [&](const ItemPos &q, uint32_t s) {
+        const uint32_t r = q.r;
+        uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[r % kYB]);
         if (pair_on) {
             float2 a0 = make_float2(0.f, 0.f), a1 = a0, b0 = a0, b1 = a0;
-            mix_pair_half(sm_a + P.off_xs + s * P.xs_bytes, sm_a + P.off_tab[tb] + wlane, kp >> 1,
-                          offs, a0, a1, b0, b1);
+            mix_pair_half(sm_a + P.off_xs + s * P.xs_bytes, sm_a + P.off_tab[r % kNT] + wlane,
+                          olane, lxx, kp >> 1, a0, a1, b0, b1);
             // lane lig's positions are lig + 32 hf + 8 m
             uint16_t *yh = ys + (lig + 32 * hf) * Es + ea;
             const int stp = kGS * Es;
@@ -765,9 +1014,9 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
                 const float av[4] = {a0.x, a0.y, a1.x, a1.y};
                 const float bv[4] = {b0.x, b0.y, b1.x, b1.y};
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    yh[q * stp] = f32_to_bf16(av[q]);
-                    if (eb < R) yh[q * stp + 1] = f32_to_bf16(bv[q]);
+                for (int m = 0; m < 4; ++m) {
+                    yh[m * stp] = f32_to_bf16(av[m]);
+                    if (eb < R) yh[m * stp + 1] = f32_to_bf16(bv[m]);
                 }
             } else {
                 uint32_t *yw = reinterpret_cast<uint32_t *>(yh);
@@ -779,37 +1028,20 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
             }
         }
         // the residual column (table role)
-        const int p0 = t * kTP, np = min(kTP, P.HW - p0);
-        if (st < np) ys[st * Es + R] = f32_to_bf16(res[rc * kTP + st]);
-        const int cnt = np * E;
-        uint16_t *dst = P.y + ((size_t)n * P.HW + p0) * E;
-        if (P.bulk_y) {
-            // [np][E] is contiguous in shared memory and in y: one bulk copy
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            bar_sync(kBarMix, kMixT);
-            if (st == 0) {
-                // the slot, the table and the residual column are read
-                mbar_arrive(mbar(P, sm, kMbEmpty + s));
-                mbar_arrive(mbar(P, sm, kMbTFree + tb));
-                mbar_arrive(mbar(P, sm, kMbRFree + rc));
-                asm volatile(
-                    "cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n\t"
-                    "cp.async.bulk.commit_group;\n\t"
-                    "cp.async.bulk.wait_group.read 1;" ::"l"(dst),
-                    "r"(smem_u32(ys)), "r"((uint32_t)cnt * 2u)
-                    : "memory");
-            }
-            continue;
-        }
-        bar_sync(kBarMix, kMixT);
-        if (st == 0) {
-            // the slot, the table and the residual column are read
-            mbar_arrive(mbar(P, sm, kMbEmpty + s));
-            mbar_arrive(mbar(P, sm, kMbTFree + tb));
-            mbar_arrive(mbar(P, sm, kMbRFree + rc));
-        }
-        // rows of y not 16-byte aligned: 16-byte streaming stores between a
-        // 16-bit head and tail
+        if (st < q.np(P)) ys[st * Es + R] = f32_to_bf16(res[(r % kRS) * kTP + st]);
+    };
+    // item q's slot, table and residual column are read
+    auto release = [&](const ItemPos &q, uint32_t s) {
+        mbar_arrive(mbar(P, sm, kMbEmpty + s));
+        mbar_arrive(mbar(P, sm, kMbTFree + q.r % kNT));
+        mbar_arrive(mbar(P, sm, kMbRFree + q.r % kRS));
+    };
+    // rows of y not 16-byte aligned: 16-byte streaming stores between a
+    // 16-bit head and tail
+    auto store_item = [&](const ItemPos &q) {
+        const uint16_t *ys = reinterpret_cast<const uint16_t *>(sm + P.off_ys[q.r % kYB]);
+        const int cnt = q.np(P) * E;
+        uint16_t *dst = P.y + ((size_t)q.n * P.HW + q.p0()) * E;
         const int head = min(
             cnt, (int)(((16u - ((uint32_t)reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u) >> 1));
         for (int o = st; o < head; o += kMixT) {
@@ -822,12 +1054,12 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
             int p = fdiv(o, E, P.inv_E), e = o - p * E;
             uint32_t w[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
+            for (int m = 0; m < 4; ++m) {
                 const uint32_t lo = ys[p * Es + e];
                 if (++e == E) { e = 0; ++p; }
                 const uint32_t hi = ys[p * Es + e];
                 if (++e == E) { e = 0; ++p; }
-                w[q] = lo | (hi << 16);
+                w[m] = lo | (hi << 16);
             }
             __stcs(reinterpret_cast<uint4 *>(dst + o), make_uint4(w[0], w[1], w[2], w[3]));
         }
@@ -835,12 +1067,76 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
             const int p = fdiv(o, E, P.inv_E);
             __stcs(dst + o, ys[p * Es + (o - p * E)]);
         }
+    };
+    // rounds of two consecutive items (the last may have one)
+    const uint32_t nb = cta_items(P);
+    FullPhase fph;
+    ItemPos q(P);
+    while (q.r < nb) {
+        ItemPos q2 = q;
+        q2.next(P);
+        const bool two = q2.r < nb;
+        const uint32_t s1 = mix_slot<F>(P, q.r, nb), s2 = two ? mix_slot<F>(P, q2.r, nb) : 0u;
+        const uint32_t fp1 = fph.take(s1), fp2 = two ? fph.take(s2) : 0u;
+        // six threads wait for the two slots, tables and residual columns at
+        // once, the others at the barrier; thread 0 has also seen the bulk
+        // copies of the previous round finish reading their ys buffers
+        bool ok = true;
+        const int wi = st >> 5;
+        if ((st & 31) == 0 && wi < (two ? 6 : 3)) {
+            const ItemPos &w = wi < 3 ? q : q2;
+            const uint32_t wr = w.r, wit = w.it;
+            const int kind = wi % 3;
+            if (kind == 0)
+                ok = ring_wait(mbar(P, sm, kMbFull + (wi < 3 ? s1 : s2)), wi < 3 ? fp1 : fp2, P.ctrl,
+                               wit);
+            else if (kind == 1)
+                ok = ring_wait(mbar(P, sm, kMbTReady + wr % kNT), (wr / kNT) & 1u, P.ctrl, wit);
+            else
+                ok = ring_wait(mbar(P, sm, kMbRDone + wr % kRS), (wr / kRS) & 1u, P.ctrl, wit);
+        }
+        if (!bar_and(kBarMix, kMixT, ok)) break;
+        mix_item(q, s1);
+        if (two) mix_item(q2, s2);
+        if (P.bulk_y) {
+            // [np][E] is contiguous in shared memory and in y: one bulk copy
+            // per item, one group per round
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            bar_sync(kBarMix, kMixT);
+            if (st == 0) {
+                release(q, s1);
+                if (two) release(q2, s2);
+                for (int i = 0; i < (two ? 2 : 1); ++i) {
+                    const ItemPos &w = i == 0 ? q : q2;
+                    uint16_t *dst = P.y + ((size_t)w.n * P.HW + w.p0()) * E;
+                    asm volatile(
+                        "cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+                        "r"(smem_u32(sm + P.off_ys[w.r % kYB])),
+                        "r"((uint32_t)(w.np(P) * E) * 2u)
+                        : "memory");
+                }
+                asm volatile(
+                    "cp.async.bulk.commit_group;\n\t"
+                    "cp.async.bulk.wait_group.read 1;" ::: "memory");
+            }
+        } else {
+            bar_sync(kBarMix, kMixT);
+            if (st == 0) {
+                release(q, s1);
+                if (two) release(q2, s2);
+            }
+            store_item(q);
+            if (two) store_item(q2);
+        }
+        q = q2;
+        if (two) q.next(P);
     }
     // bulk copies complete before the CTA exits
     if (st == 0 && P.bulk_y) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
 // ================================================================ the mix kernel
+template <bool F>
 __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P) {
     extern __shared__ __align__(128) unsigned char sm[];
     const int tid = threadIdx.x;
@@ -872,10 +1168,10 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
     }
     __syncthreads();
 
-    if (tid < kMixT) mix_role(P, sm);
-    else if (loader) load_role(P, sm, load_units(P, tid - kLoad0));
-    else if (tid < kProd0) table_role(P, sm, tag);
-    else copy_role(P, sm);
+    if (tid < kMixT) mix_role<F>(P, sm);
+    else if (loader) load_role<F>(P, sm, load_units(P, tid - kLoad0), tag);
+    else if (tid < kProd0) table_role<F>(P, sm, tag);
+    else copy_role<F>(P, sm);
 
     // the last CTA advances the epoch (the tag of the next forward)
     __syncthreads();
@@ -894,7 +1190,8 @@ __global__ void __launch_bounds__(kRingT, 1) moce_ring_kernel(const RingParams P
 struct RingPlan {
     int D = 0, CG = 0, kp = 0, Es = 0, Kg = 0;
     size_t xs_bytes = 0, off_xs = 0, off_tab[kNT] = {}, off_ys[kYB] = {};
-    size_t off_res = 0, off_rred = 0, off_U = 0, off_bar = 0, smem = 0;
+    size_t off_res = 0, off_rred = 0, off_U = 0, off_offs = 0, off_pool = 0, off_bar = 0;
+    size_t smem = 0;
 };
 
 int sm_count() {
@@ -907,7 +1204,7 @@ int sm_count() {
 // Shared memory of pass 2: D slots of C + 1 staged rows (row C = zeros), kNT
 // mixing tables, kYB output tiles, the residual partial sums, U, mbarriers.
 // D is the largest count (at most kMaxD) that fits.
-bool ring_plan(int C, int R, int k, bool bulk_y, RingPlan *plan) {
+bool ring_plan(int C, int R, int k, bool bulk_y, bool fused, RingPlan *plan) {
     if (C % 8 != 0 || C < 8 || C > 256 || k < 1 || k > kGateMaxK || R < 1 || R > 2 * kMaxPairs)
         return false;
     RingPlan p;
@@ -929,6 +1226,8 @@ bool ring_plan(int C, int R, int k, bool bulk_y, RingPlan *plan) {
     p.off_res = take((size_t)kRS * kTP * 4, 16);
     p.off_rred = take((size_t)kResParts * kTP * 4, 16);
     p.off_U = take((size_t)C * 4, 16);
+    p.off_offs = take((size_t)kWBlock * 8, 16);
+    if (fused) p.off_pool = take(sizeof(PoolSmem), 16);
     p.off_bar = take((size_t)kMbWords * 8, 8);
     const size_t fixed = align_up(off, 128);
     const size_t budget = 227 * 1024;
@@ -942,17 +1241,17 @@ bool ring_plan(int C, int R, int k, bool bulk_y, RingPlan *plan) {
 
 }  // namespace
 
-bool ring_supported(int N, int HW, int C, int R, int k) {
+bool ring_supported(int N, int HW, int C, int R, int k, bool fused) {
     (void)N;
     RingPlan plan;
-    return HW >= 1 && ring_plan(C, R, k, false, &plan);
+    return HW >= 1 && ring_plan(C, R, k, false, fused, &plan);
 }
 
 cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
                         const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
                         const float *W1, const float *b1, const float *w2, const float *b2,
                         float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
-                        cudaStream_t s) {
+                        bool fused, cudaStream_t s) {
     const int G = sm_count();
     if (G < 1) return cudaErrorInvalidDevice;
     // every output tile [np][R + 1] starts and ends on a 16-byte boundary of y
@@ -960,7 +1259,7 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     const bool bulk_y =
         ((long long)HW * (R + 1)) % 8 == 0 && (reinterpret_cast<uintptr_t>(y) & 15u) == 0;
     RingPlan plan;
-    if (!ring_plan(C, R, k, bulk_y, &plan)) return cudaErrorNotSupported;
+    if (!ring_plan(C, R, k, bulk_y, fused, &plan)) return cudaErrorNotSupported;
     const int T = (HW + kTP - 1) / kTP;
     const unsigned long long items = (unsigned long long)N * T;
     if (items >= 0xffff0000ull) return cudaErrorInvalidValue;
@@ -992,9 +1291,15 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     Q.tau = reinterpret_cast<float *>(ws + L.tau);
     Q.kp = plan.kp;
     Q.Kg = plan.Kg;
+    cudaError_t err = cudaSuccess;
+    if (fused) {
+        // single pass: every tile is its own run
+        Q.RL = 1;
+        Q.RPE = T;
+        Q.runs = (uint32_t)items;
+    } else {
     int per_sm = 0;
-    cudaError_t err =
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, moce_poolgate_kernel, kPoolT, 0);
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, moce_poolgate_kernel, kPoolT, 0);
     if (err != cudaSuccess) return err;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // runs of RL tiles: about one resident wave of CTAs, at most 255 runs per
@@ -1012,8 +1317,9 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     moce_poolgate_kernel<<<(unsigned)g1, kPoolT, 0, s>>>(Q);
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
+    }
 
-    // pass 2: mixing
+    // pass 2 (or the single pass): mixing
     RingParams P;
     P.x = x;
     P.y = y;
@@ -1043,16 +1349,34 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     P.off_rred = (uint32_t)plan.off_rred;
     P.inv_nU = nU > 0 ? 1.0f / (float)nU : 0.0f;
     P.off_U = (uint32_t)plan.off_U;
+    P.off_offs = (uint32_t)plan.off_offs;
     P.off_bar = (uint32_t)plan.off_bar;
     P.inv_E = 1.0f / (float)(R + 1);
-    if ((err = cudaFuncSetAttribute(moce_ring_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const void *kern = fused ? reinterpret_cast<const void *>(moce_ring_kernel<true>)
+                             : reinterpret_cast<const void *>(moce_ring_kernel<false>);
+    if ((err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     (int)plan.smem)) != cudaSuccess)
         return err;
     const unsigned g2 = (unsigned)std::min<unsigned long long>(items, (unsigned long long)G);
     P.Gn = (int)(g2 / (unsigned)T);
     P.Gt = (int)(g2 % (unsigned)T);
-    moce_ring_kernel<<<g2, kRingT, plan.smem, s>>>(P);
-    return cudaGetLastError();
+    P.lead = kLead;
+    P.off_pool = (uint32_t)plan.off_pool;
+    P.pool = Q;
+    if (!fused) {
+        moce_ring_kernel<false><<<g2, kRingT, plan.smem, s>>>(P);
+        return cudaGetLastError();
+    }
+    // CTAs wait for gates that other CTAs of the launch run: all of them
+    // must be resident (one per SM), which a cooperative launch guarantees
+    int per_sm = 0;
+    if ((err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, moce_ring_kernel<true>, kRingT,
+                                                             plan.smem)) != cudaSuccess)
+        return err;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    void *args[] = {&P};
+    return cudaLaunchCooperativeKernel(kern, dim3(g2),
+                                       dim3(kRingT), args, plan.smem, s);
 }
 
 }  // namespace moce

@@ -106,6 +106,7 @@ def test_forward_path_selection_on_host(lib):
                  0.2, 6.0, fake, fake, ws_bytes, path, None)
 
     assert call(1, 7) == 1             # not a path
+    assert call(0, 5) == 3             # nor a single-pass ring kernel
     assert call(1, -1) == 1
     assert call(0, 2) == 3             # fp32 has no two-pass kernel: unsupported, nothing enqueued
     assert call(0, 1) == 3             # nor a pipeline kernel
@@ -115,6 +116,8 @@ def test_forward_path_selection_on_host(lib):
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == 2
     assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == b"moce_poolgate_kernel+moce_ring_kernel"
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 3) == 1
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 5) == 1
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 5) == b"moce_ring_kernel"
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
     assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == b"pool+gate+mix"
     # misaligned x or NCHW leaves only the step kernels
