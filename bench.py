@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="auto",
+                    help="kernel path of the forward (auto, two_pass, pipe, ring, fused, steps)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline leg")
     return ap.parse_args()
@@ -88,15 +90,15 @@ def csrc_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload: str):
-    """DRAM bytes per launch from a committed ncu summary, if taken on the current kernels."""
+def ncu_traffic(workload: str, kernel: str):
+    """DRAM bytes per step from a committed ncu summary, if taken on the current kernels."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         d = json.load(f)
     rec = d.get(workload)
-    if not rec or rec.get("csrc_hash") != csrc_hash():
+    if not rec or rec.get("csrc_hash") != csrc_hash() or rec.get("kernel", kernel) != kernel:
         return None
     return rec.get("dram_bytes_per_launch")
 
@@ -286,9 +288,9 @@ def run_ours(args, cfg):
           for _ in range(n_rot)]
     ws = moce.Workspace(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k, device=dev)
     fwd = lambda i: moce.moce_forward(xs[i % n_rot], "nhwc", packed, W1, b1, w2, b2, cfg.tau_min,
-                                      cfg.tau_max, ws=ws, y=ys[i % n_rot])
-    launches_per_step = moce.moce_forward_launches(xs[0], "nhwc", cfg.C_out, cfg.k)
-    kernel_name = moce.moce_forward_kernel(xs[0], "nhwc", cfg.C_out, cfg.k)
+                                      cfg.tau_max, ws=ws, y=ys[i % n_rot], path=args.path)
+    launches_per_step = moce.moce_forward_launches(xs[0], "nhwc", cfg.C_out, cfg.k, path=args.path)
+    kernel_name = moce.moce_forward_kernel(xs[0], "nhwc", cfg.C_out, cfg.k, path=args.path)
 
     for i in range(args.warmup):
         fwd(i)
@@ -336,7 +338,7 @@ def run_ours(args, cfg):
     kern_s = statistics.mean(launch_ms) * 1e-3
     achieved = nbytes / kern_s / 1e9
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / peaks["hbm_gbs"], "traffic": ncu_traffic(cfg.name),
+                "frac": achieved / peaks["hbm_gbs"], "traffic": ncu_traffic(cfg.name, kernel_name),
                 "peak_source": f"{peak_src} (burst copy)", "kernel": (
                     kernel_name if launches_per_step == 1 else
                     f"{kernel_name} ({launches_per_step} launches)"),
@@ -366,14 +368,14 @@ def run_ours(args, cfg):
     for _ in range(3):
         x_dev.copy_(x_host, non_blocking=True)
         moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
-                          y=y_dev)
+                          y=y_dev, path=args.path)
         y_host.copy_(y_dev, non_blocking=True)
     torch.cuda.synchronize()
     e0.record()
     for _ in range(Ke):
         x_dev.copy_(x_host, non_blocking=True)
         moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
-                          y=y_dev)
+                          y=y_dev, path=args.path)
         y_host.copy_(y_dev, non_blocking=True)
     e1.record()
     torch.cuda.synchronize()
@@ -401,6 +403,7 @@ def run_ours(args, cfg):
                                     "activations)",
             "config": {"workload": cfg.name, "N": cfg.N, "H": cfg.H, "W": cfg.W,
                        "C_in": cfg.C_in, "C_out": cfg.C_out, "k": cfg.k, "n_resid": packed.n_resid,
+                       "path": kernel_name,
                        "storage_dtype": "bf16", "layout": "nhwc",
                        "l2": f"inputs rotate over {n_rot} copies ({n_rot * x_bytes / 2**20:.0f} MiB"
                              f" > 3x the {l2 / 2**20:.0f} MiB L2)",

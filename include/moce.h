@@ -62,6 +62,7 @@ typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
  * the same layer (Sec. 3.2-3.4) and gives the same results within bf16
  * output rounding; they differ in how x travels through the GPU.
  *   MOCE_PATH_AUTO      the fastest path that supports the arguments
+ *                       (TWO_PASS, else PIPE, else FUSED, else STEPS)
  *   MOCE_PATH_PIPE      one warp-specialised persistent kernel (NHWC bf16,
  *                       8 <= C_in <= 256, C_in % 8 == 0, k <= 16)
  *   MOCE_PATH_TWO_PASS  a pooling+gate kernel, then a mixing kernel that
@@ -185,9 +186,10 @@ moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
  *   ws, ws_bytes: >= moce_workspace_bytes(N, H, W, C_in, C_out, k), 256-byte
  *   aligned, zero-filled before its first use (moce_workspace_init); one
  *   workspace serves one stream at a time.
- * NHWC bf16 with C_in % 8 == 0 and 16-byte aligned x runs one fused
- * persistent kernel; other layouts/dtypes run a sequence of kernels (the
- * choice is moce_forward_path's MOCE_PATH_AUTO).
+ * NHWC bf16 with C_in % 8 == 0 and 16-byte aligned x runs the two-pass
+ * path where it fits (C_in <= 256, C_out <= 64, k <= 16), else a persistent
+ * kernel; other layouts/dtypes run a sequence of kernels (the choice is
+ * moce_forward_path's MOCE_PATH_AUTO).
  * Asynchronous; device-side failures of the fused kernels (a bounded wait
  * that ran out) are reported by moce_check_device_error.
  */
@@ -248,10 +250,11 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
 
 /*
  * Name of the kernel path moce_forward takes for these arguments:
- * "moce_pipe_kernel" (the warp-specialised pipeline, NHWC bf16 with
- * C_in <= 256), "moce_fused_kernel" (the two-group persistent kernel) or
- * "pool+gate+mix" (one kernel per step). NULL for arguments moce_forward
- * would reject. Enqueues nothing; the string is static.
+ * "moce_poolgate_kernel+moce_ring_kernel" (the two-pass path),
+ * "moce_pipe_kernel" (the warp-specialised pipeline), "moce_fused_kernel"
+ * (the two-group persistent kernel) or "pool+gate+mix" (one kernel per
+ * step). NULL for arguments moce_forward would reject. Enqueues nothing; the
+ * string is static.
  */
 const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                 moce_dtype_t dtype, moce_layout_t layout);

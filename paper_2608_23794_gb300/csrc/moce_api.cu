@@ -140,8 +140,9 @@ static moce_path_t pick_path(const void *x, int N, int HW, int C_in, int C_out, 
     const bool ring = vec && ring_supported(N, HW, C_in, C_out, k, true);
     const bool fused = vec && fused_supported(N, HW, C_in, C_out, k);
     switch (want) {
-        case MOCE_PATH_AUTO:
-            return pipe ? MOCE_PATH_PIPE : fused ? MOCE_PATH_FUSED : MOCE_PATH_STEPS;
+        case MOCE_PATH_AUTO:  // the fastest measured first
+            return two ? MOCE_PATH_TWO_PASS
+                       : pipe ? MOCE_PATH_PIPE : fused ? MOCE_PATH_FUSED : MOCE_PATH_STEPS;
         case MOCE_PATH_PIPE: return pipe ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_TWO_PASS: return two ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_FUSED: return fused ? want : MOCE_PATH_AUTO;

@@ -367,6 +367,9 @@ __global__ void __launch_bounds__(kPoolT) moce_poolgate_kernel(const PoolParams 
     const bool own = 8 * cb < P.C;
     const uint32_t tag = ld_relaxed(P.ctrl + kCtrlEpoch) + 1u;
     const uint32_t drop = ld_relaxed(P.ctrl + kCtrlDropItem);
+    // the mixing pass may launch now: it reads pass 1's results only after
+    // griddepcontrol.wait, and the epoch only at its end
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     for (uint32_t ru = blockIdx.x; ru < P.runs; ru += gridDim.x) {
         const int n = (int)(ru / (uint32_t)P.RPE), j = (int)(ru - (uint32_t)n * P.RPE);
         const int t0 = j * P.RL, t1 = min(P.T, t0 + P.RL);
@@ -816,6 +819,9 @@ __device__ void table_role(const RingParams &P, unsigned char *sm, uint32_t tag)
     uint32_t wcopies = 0;
     bool wok = true;
     if (tt == 0) {
+        // a two-pass launch may start before pass 1 has finished; the
+        // weights and tags are read after it has
+        if (!F) asm volatile("griddepcontrol.wait;" ::: "memory");
         for (int i = 0; i < 2 && wok && wq.r < nb; ++i) {
             wok = made_wait<F>(P, wq.n, tag, read_tag<F>(P, wq.n), wq.it);
             if (wok) weights_copy(P, sm, wq), ++wcopies, wq.next(P);
@@ -1364,8 +1370,19 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
     P.off_pool = (uint32_t)plan.off_pool;
     P.pool = Q;
     if (!fused) {
-        moce_ring_kernel<false><<<g2, kRingT, plan.smem, s>>>(P);
-        return cudaGetLastError();
+        // programmatic dependent launch: the CTAs start on SMs that pass 1
+        // has left and stage x while pass 1 finishes
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(g2);
+        cfg.blockDim = dim3(kRingT);
+        cfg.dynamicSmemBytes = plan.smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, moce_ring_kernel<false>, P);
     }
     // CTAs wait for gates that other CTAs of the launch run: all of them
     // must be resident (one per SM), which a cooperative launch guarantees

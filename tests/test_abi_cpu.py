@@ -111,8 +111,9 @@ def test_forward_path_selection_on_host(lib):
     assert call(0, 2) == 3             # fp32 has no two-pass kernel: unsupported, nothing enqueued
     assert call(0, 1) == 3             # nor a pipeline kernel
     # bf16 NHWC, aligned x: every path runs these shapes
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 1
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"moce_pipe_kernel"
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 2   # the fastest: two-pass
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"moce_poolgate_kernel+moce_ring_kernel"
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 1) == b"moce_pipe_kernel"
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == 2
     assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == b"moce_poolgate_kernel+moce_ring_kernel"
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 3) == 1
@@ -125,9 +126,10 @@ def test_forward_path_selection_on_host(lib):
     assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 1) == 0
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 2) == 0
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3
-    # more experts than the two-pass kernel's pairs
+    # more experts than the two-pass kernel's pairs: the pipeline kernel
     assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 2) == 0
     assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 1) == 1
+    assert name(fake, 2, 8, 8, 256, 96, 4, 1, 0, 0) == b"moce_pipe_kernel"
 
 
 def test_pack_rejects_bad_arguments_on_host(lib):
