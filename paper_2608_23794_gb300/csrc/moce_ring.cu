@@ -23,16 +23,16 @@
 // four lane groups of a mixing warp (pairs 8 apart) read different banks.
 //
 // Pass 2, moce_ring_kernel, reads x again and mixes it: one CTA per SM takes
-// items b, b + G, ...; its copy warp (27) brings each tile (64 positions x C
+// items b, b + G, ...; its copy warp (19) brings each tile (64 positions x C
 // channels, contiguous in NHWC) into a ring of D shared-memory slots by one
 // bulk copy as soon as a slot is free, so several tiles are in flight; the
-// load warps (16-23) transpose a landed tile in place to channel-major rows;
-// the table warps (24-26) bring the weights of the item two ahead into one of
+// load warps (8-15) transpose a landed tile in place to channel-major rows;
+// the table warps (16-18) bring the weights of the item two ahead into one of
 // six mixing tables by a bulk copy and sum the tile's unselected channels for
-// the residual expert (Eq. (res)); the mix warps (0-15) mix two items per
+// the residual expert (Eq. (res)); the mix warps (0-7) mix two items per
 // round, each slot with its table: each group of 8 lanes owns one expert pair
-// and half of every 16-byte row chunk (4 positions per lane) for the whole
-// launch, with the pair's row offsets in registers (Eq. (expert)); each tile
+// for the whole launch and reads one 16-byte row chunk (8 positions) per lane
+// and support, with the pair's row offsets in a shared table (Eq. (expert)); each tile
 // of y, residual column included, leaves by one bulk copy. The roles hand
 // slots and tables over through shared-memory mbarriers; every wait is
 // bounded and none crosses CTAs. No role holds global loads in registers
@@ -49,10 +49,10 @@ constexpr int kTP = kRingTile;        // positions per tile
 constexpr int kGS = 8;                // lanes of a mixing group
 constexpr int kRB = 16 * kGS;         // bytes per staged channel row (kTP bf16)
 constexpr int kFM = 7;                // chunk swizzle mask of the staged rows
-constexpr int kMixT = 512;            // pass 2: mix warps 0-15
-constexpr int kLoadT = 256;           // pass 2: load warps 16-23
-constexpr int kTabT = 96;             // pass 2: table warps 24-26
-constexpr int kProdT = 32;            // pass 2: the copy warp 27
+constexpr int kMixT = 256;            // pass 2: mix warps 0-7
+constexpr int kLoadT = 256;           // pass 2: load warps 8-15
+constexpr int kTabT = 96;             // pass 2: table warps 16-18
+constexpr int kProdT = 32;            // pass 2: the copy warp 19
 constexpr int kLoadW = kLoadT / 32;
 constexpr int kLU = 32 / kLoadW;      // staging units per load thread and tile (at C = 256)
 constexpr int kRingT = kMixT + kLoadT + kTabT + kProdT;
@@ -60,7 +60,7 @@ constexpr int kLoad0 = kMixT;                    // first load thread
 constexpr int kTab0 = kMixT + kLoadT;            // first table thread
 constexpr int kProd0 = kTab0 + kTabT;            // the copy warp's first thread
 constexpr int kResParts = kTabT / 8;             // residual: U entries split kResParts ways
-constexpr int kPairWarps = 8;         // mix warps w and w + 8 share expert pairs
+constexpr int kPairWarps = 8;         // mix warp w takes expert pairs w + 8 h
 // Mixing tables: the weights of item r + 2 go into table (r + 2) mod kNT as
 // the table role starts item r, which must then wait only for items the mix
 // role has finished (r - 3 and before: a mixing round takes two items), so
@@ -74,8 +74,8 @@ constexpr int kGateMaxK = 16;          // support positions a mixing lane keeps 
 constexpr int kMaxPairs = 32;          // expert pairs: one per mixing group
 constexpr int kWBlock = kMaxPairs * 8; // float4 entries of a weight block
 constexpr int kBarMix = 1, kBarLoad = 2, kBarTab = 3;
-// Registers per thread: 72 for every role (kRingT * 72 <= 65536).
-constexpr int kLaunchRegs = 72, kMixRegs = 72, kLoadRegs = 72, kTabRegs = 72;
+// Registers per thread: 96 for every role (kRingT * 96 <= 65536).
+constexpr int kLaunchRegs = 96, kMixRegs = 96, kLoadRegs = 96, kTabRegs = 96;
 static_assert(kMixT * kMixRegs + kLoadT * kLoadRegs + (kTabT + kProdT) * kTabRegs <=
                   kRingT * kLaunchRegs,
               "register split exceeds the launch allocation");
@@ -85,7 +85,7 @@ constexpr int kPoolT = 256;           // pass 1 threads per CTA
 constexpr int kPoolCTAs = 8;          // pass 1 CTAs per SM
 constexpr int kAccG = 4;              // accumulator words per (example, channel)
 static_assert(kRingT * kLaunchRegs <= 65536, "launch registers at one CTA per SM");
-static_assert(kMixT == 2 * kPairWarps * 32, "two mix warps per set of expert pairs");
+static_assert(kMixT == kPairWarps * 32, "one mix warp per set of expert pairs");
 static_assert(kTP == 8 * kGS, "a group's lanes cover the tile");
 static_assert(kPoolT == 4 * kTP, "pass 1: 32 channel blocks x 8 rows of positions");
 
@@ -911,52 +911,58 @@ __device__ __forceinline__ float2 unpack2_split(uint32_t w) {
     return make_float2(__uint_as_float(lo), __uint_as_float(w & 0xffff0000u));
 }
 
-// Weighted sums of the lane's expert pair for its 4 positions. Entry i2 of
-// the pair is one float4 of weights (at wa + 512 i2) and four 8-byte halves
-// of row chunks at xa + the 16-bit offsets of the pair's offset word
-// (at oa + 256 i2: {expert a, expert b}, support positions 2 i2 and 2 i2 + 1
-// in the low and high half, XORed with the lane's chunk and half, lxx).
-// Entry i2 + 1's reads are issued before entry i2 is added and the offsets
-// two entries ahead, so a lane keeps shared-memory reads in flight while it
-// computes.
-struct MixEntry {
+
+// Weighted sums of the lane's expert pair for its 8 positions (the 16-byte
+// chunk of each row): entry i2 is one float4 of weights (at wa + 512 i2) and
+// four row chunks at xa + the 16-bit offsets of the pair's offset word (at
+// oa + 256 i2, XORed with the lane's chunk, lxx); acc[j] (expert a) and
+// acc[4 + j] (expert b) hold word j's positions lig + 16 j and lig + 16 j + 8.
+// Entry i2 + 1's reads are issued before entry i2 is added.
+__device__ __forceinline__ uint4 lds128u(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(a));
+    return v;
+}
+struct MixEntry8 {
     float4 w;
-    uint2 a0, a1, b0, b1;
+    uint4 a0, a1, b0, b1;
 };
-__device__ __forceinline__ MixEntry mix_load(uint32_t xa, uint32_t wa, uint2 o, uint32_t lxx,
-                                             int i2) {
-    MixEntry m;
+__device__ __forceinline__ MixEntry8 mix_load8(uint32_t xa, uint32_t wa, uint2 o, uint32_t lxx,
+                                               int i2) {
+    MixEntry8 m;
     const uint32_t oa = o.x ^ lxx, ob = o.y ^ lxx;
     m.w = lds128f(wa + 512u * i2);
-    m.a0 = lds64(xa + (oa & 0xffffu));
-    m.a1 = lds64(xa + (oa >> 16));
-    m.b0 = lds64(xa + (ob & 0xffffu));
-    m.b1 = lds64(xa + (ob >> 16));
+    m.a0 = lds128u(xa + (oa & 0xffffu));
+    m.a1 = lds128u(xa + (oa >> 16));
+    m.b0 = lds128u(xa + (ob & 0xffffu));
+    m.b1 = lds128u(xa + (ob >> 16));
     return m;
 }
-__device__ __forceinline__ void mix_pair_half(uint32_t xa, uint32_t wa, uint32_t oa,
-                                              uint32_t lxx, int npairs, float2 &a0, float2 &a1,
-                                              float2 &b0, float2 &b1) {
+__device__ __forceinline__ void mix_add4(float2 *acc, float w, const uint4 &v) {
+    const float2 ww = make_float2(w, w);
+    acc[0] = __ffma2_rn(ww, unpack2_split(v.x), acc[0]);
+    acc[1] = __ffma2_rn(ww, unpack2_split(v.y), acc[1]);
+    acc[2] = __ffma2_rn(ww, unpack2_split(v.z), acc[2]);
+    acc[3] = __ffma2_rn(ww, unpack2_split(v.w), acc[3]);
+}
+__device__ __forceinline__ void mix_pair_full(uint32_t xa, uint32_t wa, uint32_t oa, uint32_t lxx,
+                                              int npairs, float2 *acc) {
     uint2 on = lds64(oa + 256u);
-    MixEntry cur = mix_load(xa, wa, lds64(oa), lxx, 0);
+    MixEntry8 cur = mix_load8(xa, wa, lds64(oa), lxx, 0);
 #pragma unroll
     for (int i2 = 0; i2 < kGateMaxK / 2; ++i2) {
         if (i2 >= npairs) break;
-        MixEntry nxt = cur;
+        MixEntry8 nxt = cur;
         if (i2 + 1 < kGateMaxK / 2 && i2 + 1 < npairs) {
-            nxt = mix_load(xa, wa, on, lxx, i2 + 1);
+            nxt = mix_load8(xa, wa, on, lxx, i2 + 1);
             if (i2 + 2 < kGateMaxK / 2 && i2 + 2 < npairs) on = lds64(oa + 256u * (i2 + 2));
         }
-        const float2 wa0 = make_float2(cur.w.x, cur.w.x), wa1 = make_float2(cur.w.y, cur.w.y);
-        const float2 wb0 = make_float2(cur.w.z, cur.w.z), wb1 = make_float2(cur.w.w, cur.w.w);
-        a0 = __ffma2_rn(wa0, unpack2_split(cur.a0.x), a0);
-        a1 = __ffma2_rn(wa0, unpack2_split(cur.a0.y), a1);
-        b0 = __ffma2_rn(wb0, unpack2_split(cur.b0.x), b0);
-        b1 = __ffma2_rn(wb0, unpack2_split(cur.b0.y), b1);
-        a0 = __ffma2_rn(wa1, unpack2_split(cur.a1.x), a0);
-        a1 = __ffma2_rn(wa1, unpack2_split(cur.a1.y), a1);
-        b0 = __ffma2_rn(wb1, unpack2_split(cur.b1.x), b0);
-        b1 = __ffma2_rn(wb1, unpack2_split(cur.b1.y), b1);
+        mix_add4(acc, cur.w.x, cur.a0);
+        mix_add4(acc + 4, cur.w.z, cur.b0);
+        mix_add4(acc, cur.w.y, cur.a1);
+        mix_add4(acc + 4, cur.w.w, cur.b1);
         cur = nxt;
     }
 }
@@ -970,14 +976,10 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
     const uint32_t lx = (uint32_t)lig << 4;
     const int R = P.R, E = R + 1, kp = P.kp, NP = (R + 1) >> 1, Es = P.Es;
     const float *res = reinterpret_cast<const float *>(sm + P.off_res);
-    // this group's expert pair (warps w and w + 8 take pairs (w mod 8) + 8h)
-    // and half hf of each 16-byte chunk (positions lig + 32 hf + 8 m, m < 4):
-    // the groups of a warp alternate halves, so a warp's 8-byte reads of four
-    // rows hit every bank twice; row offsets are fixed for the whole launch;
-    // padding positions and the twin of an odd last expert read the zero row
-    // (their weights are 0)
-    const int pr = (warp & (kPairWarps - 1)) + kPairWarps * h;
-    const int hf = (h & 1) ^ (warp / kPairWarps);
+    // this group's expert pair (warp w's groups take pairs w + 8 h); padding
+    // positions and the twin of an odd last expert read the zero row (their
+    // weights are 0)
+    const int pr = warp + kPairWarps * h;
     const int ea = 2 * pr, eb = ea + 1;
     const bool pair_on = pr < NP;
     // the offset table: entry (pair p, i2) at wslot(p, i2), two words of
@@ -998,7 +1000,7 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
         ot[wslot(p, i2)] = make_uint2(o[0] | (o[1] << 16), o[2] | (o[3] << 16));
     }
     bar_sync(kBarMix, kMixT);
-    const uint32_t lxx = (lx | ((uint32_t)hf << 3)) * 0x10001u;
+    const uint32_t lxx = lx * 0x10001u;
     const uint32_t wlane = 16u * (uint32_t)(4 * (pr & 7) + (pr >> 3));  // wslot(pr, 0) * 16
     const uint32_t olane = sm_a + P.off_offs + 8u * (uint32_t)(4 * (pr & 7) + (pr >> 3));
     // item q: mix the slot with its table into ys[q.r mod kYB] and add the
@@ -1007,30 +1009,34 @@ __device__ void mix_role(const RingParams &P, unsigned char *sm) {
         const uint32_t r = q.r;
         uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys[r % kYB]);
         if (pair_on) {
-            float2 a0 = make_float2(0.f, 0.f), a1 = a0, b0 = a0, b1 = a0;
-            mix_pair_half(sm_a + P.off_xs + s * P.xs_bytes, sm_a + P.off_tab[r % kNT] + wlane,
-                          olane, lxx, kp >> 1, a0, a1, b0, b1);
-            // lane lig's positions are lig + 32 hf + 8 m
-            uint16_t *yh = ys + (lig + 32 * hf) * Es + ea;
+            float2 acc[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] = make_float2(0.f, 0.f);
+            mix_pair_full(sm_a + P.off_xs + s * P.xs_bytes, sm_a + P.off_tab[r % kNT] + wlane,
+                          olane, lxx, kp >> 1, acc);
+            // lane lig's positions are lig + 8 m: acc[m / 2], half m mod 2
+            uint16_t *yh = ys + lig * Es + ea;
             const int stp = kGS * Es;
             if (P.bulk_y || eb == R) {
                 // rows of odd length (or, for odd R, the twin's column is the
                 // residual column, written below by another thread): 16-bit
                 // stores
-                const float av[4] = {a0.x, a0.y, a1.x, a1.y};
-                const float bv[4] = {b0.x, b0.y, b1.x, b1.y};
 #pragma unroll
-                for (int m = 0; m < 4; ++m) {
-                    yh[m * stp] = f32_to_bf16(av[m]);
-                    if (eb < R) yh[m * stp + 1] = f32_to_bf16(bv[m]);
+                for (int m = 0; m < 8; ++m) {
+                    const float va = (m & 1) ? acc[m >> 1].y : acc[m >> 1].x;
+                    const float vb = (m & 1) ? acc[4 + (m >> 1)].y : acc[4 + (m >> 1)].x;
+                    yh[m * stp] = f32_to_bf16(va);
+                    if (eb < R) yh[m * stp + 1] = f32_to_bf16(vb);
                 }
             } else {
                 uint32_t *yw = reinterpret_cast<uint32_t *>(yh);
                 const int sw = stp >> 1;
-                yw[0 * sw] = pack_bf16x2(a0.x, b0.x);
-                yw[1 * sw] = pack_bf16x2(a0.y, b0.y);
-                yw[2 * sw] = pack_bf16x2(a1.x, b1.x);
-                yw[3 * sw] = pack_bf16x2(a1.y, b1.y);
+#pragma unroll
+                for (int m = 0; m < 8; ++m) {
+                    const float va = (m & 1) ? acc[m >> 1].y : acc[m >> 1].x;
+                    const float vb = (m & 1) ? acc[4 + (m >> 1)].y : acc[4 + (m >> 1)].x;
+                    yw[m * sw] = pack_bf16x2(va, vb);
+                }
             }
         }
         // the residual column (table role)
