@@ -1,17 +1,17 @@
-// Two-pass forward of a MoCE layer (Sec. 3.3-3.4) for NHWC bf16 layers with
-// C_in <= 256, C_out <= 64 and k <= 16.
+// Two-pass and single-pass ring forwards of a MoCE layer (Sec. 3.3-3.4) for
+// NHWC bf16 layers with C_in <= 256, C_out <= 64 and k <= 16.
 //
 // Every expert's temperature depends on the whole-image average of its
 // support (Sec. 3.3), so no position of an example can be mixed before all
 // of the example has been pooled. The examples are cut into tiles of 64
 // positions (tile t of example n is item n*T + t).
 //
-// Pass 1, moce_poolgate_kernel, streams x once at full bandwidth: each CTA
-// reduces a tile to its channel sums and adds them, as 64-bit fixed-point
+// Pass 1, moce_poolgate_kernel, streams x once: each CTA reduces a run of
+// tiles to its channel sums and adds them, as 64-bit fixed-point
 // integers, into accumulator words of the example (integer sums do not
 // depend on the order of the additions, so z is deterministic; a sum beyond
 // the fixed-point range is kept as an epoch-tagged fp32 word instead). The
-// CTA that counts an example's last tile reads z, evaluates the gate of
+// CTA that counts an example's last run reads z, evaluates the gate of
 // every expert (Eq. (tau)) and the softmax weights (Eq. (weights)) and
 // writes them in mixing-table order; it also clears the example's
 // accumulators for the next forward.
@@ -38,6 +38,13 @@
 // bounded and none crosses CTAs. No role holds global loads in registers
 // across a barrier: x and the weights arrive by bulk copies, so the barriers
 // never wait for HBM.
+//
+// The single-pass mode (moce_ring_kernel<true>, one cooperative launch) runs
+// pass 1's work inside the same CTAs: each CTA pools its own tiles kLead
+// rounds before it mixes them (Seq), the load warps reduce a pooled tile and
+// the CTA that counts an example's last tile runs its gate (pool_tile,
+// gate_if_last), and the table warps wait, bounded, for the example's tag
+// before they bring its weights.
 #include <algorithm>
 
 #include "moce_device.cuh"
