@@ -283,6 +283,7 @@ struct PoolSmem {
     float b1[32];
     float w2[33];
     uint32_t last;
+    uint32_t cmd;  // single pass: the load role's next step while it waits for a slot
 };
 
 // The example's gate, by the kPoolT threads (tid = 0 .. kPoolT - 1, meeting at
@@ -753,18 +754,47 @@ __device__ void load_role(const RingParams &P, unsigned char *sm, const LoadUnit
     Seq<F> q(P);
     for (; q.live(); q.next(P)) {
         const uint32_t s = q.s;
-        bool ok = true;
-        if (lt == 0) ok = ring_wait(mbar(P, sm, kMbRaw + s), q.ph, P.ctrl, q.item().it);
-        if (!bar_and(kBarLoad, kLoadT, ok)) return;
-        // the older pending count is looked at every position (the last
-        // pooled tiles' gates must not wait for the end of the sequence:
-        // mixing positions after them may need those examples)
-        unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
         if constexpr (F) {
+            // pending counts are looked at before and while the role waits
+            // for the slot: an example's gate must not wait for this CTA's
+            // slots (mixing positions of other CTAs may need the example)
             if (pend0 >= 0) gate_if_last(P, sm, pend0, old0, tag);
             pend0 = pend1;
             old0 = old1;
             pend1 = -1;
+            PoolSmem &S = *reinterpret_cast<PoolSmem *>(sm + P.off_pool);
+            for (uint32_t polls = 1;; ++polls) {
+                if (lt == 0) {
+                    uint32_t cmd = 0;  // 0: wait on, 1: landed, 2: gate pend0 now, 3: give up
+                    if (mbar_try(mbar(P, sm, kMbRaw + s), q.ph)) {
+                        cmd = 1;
+                    } else if (polls >= kSpinLimit) {
+                        report_timeout(P.ctrl, q.item().it);
+                        cmd = 3;
+                    } else if ((polls & 15u) == 0u && ld_relaxed(P.ctrl + kCtrlError) != 0u) {
+                        cmd = 3;
+                    } else if (pend0 >= 0 && polls >= 2) {
+                        cmd = 2;
+                    }
+                    S.cmd = cmd;
+                }
+                bar_sync(kBarLoad, kLoadT);
+                const uint32_t cmd = S.cmd;
+                bar_sync(kBarLoad, kLoadT);  // the command word is free again
+                if (cmd == 1) break;
+                if (cmd == 3) return;
+                if (cmd == 2) {
+                    gate_if_last(P, sm, pend0, old0, tag);
+                    pend0 = -1;
+                }
+            }
+        } else {
+            bool ok = true;
+            if (lt == 0) ok = ring_wait(mbar(P, sm, kMbRaw + s), q.ph, P.ctrl, q.item().it);
+            if (!bar_and(kBarLoad, kLoadT, ok)) return;
+        }
+        unsigned char *xs = sm + P.off_xs + s * P.xs_bytes;
+        if constexpr (F) {
             if (q.is_pool) {
                 old1 = 0xffffffffu;
                 pool_tile(P, sm, xs, q.pool, s, tag, drop, old1);
