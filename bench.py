@@ -222,7 +222,8 @@ def run_reference(args, cfg):
     per_step = 120.0 / max(1, args.steps + args.warmup)
     n_ex = int(max(1, min(cfg.N, per_step / t_ex)))
     h_rows = cfg.H if t_ex <= per_step else int(max(1, cfg.H * per_step / t_ex))
-    xs = lay.x[:n_ex, :h_rows].copy()
+    # rows are axis 1 of NHWC and axis 2 of NCHW
+    xs = (lay.x[:n_ex, :h_rows] if cfg.layout == "nhwc" else lay.x[:n_ex, :, :h_rows]).copy()
     for _ in range(args.warmup):
         oracle.forward(xs, cfg.layout, *args_o)
     t0 = time.perf_counter()
