@@ -73,9 +73,10 @@ typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
  *   MOCE_PATH_STEPS     one kernel per step: pool, gate, mix (any layout
  *                       and dtype)
  *   MOCE_PATH_RING      one cooperative kernel in which every CTA pools its
- *                       tiles a few rounds before it mixes them, the CTA
- *                       that pools an example's last tile runs the gate, and
- *                       the second read of x comes from L2 (as TWO_PASS)
+ *                       tiles a few rounds before it mixes them and the CTA
+ *                       that pools an example's last tile runs the gate
+ *                       (the shapes of TWO_PASS; correct, but slower than
+ *                       TWO_PASS on the measured workloads)
  */
 typedef enum moce_path {
     MOCE_PATH_AUTO = 0,
