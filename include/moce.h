@@ -77,6 +77,11 @@ typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
  *                       that pools an example's last tile runs the gate
  *                       (the shapes of TWO_PASS; correct, but slower than
  *                       TWO_PASS on the measured workloads)
+ *   MOCE_PATH_STREAM    one cooperative kernel that reads x from HBM once:
+ *                       each tile stays in shared memory from its pooling
+ *                       until its example's gate has run (NHWC bf16,
+ *                       64 <= C_in <= 256, C_in % 64 == 0, C_out <= 64,
+ *                       k <= 16, x 16-byte aligned)
  */
 typedef enum moce_path {
     MOCE_PATH_AUTO = 0,
@@ -84,7 +89,8 @@ typedef enum moce_path {
     MOCE_PATH_TWO_PASS = 2,
     MOCE_PATH_FUSED = 3,
     MOCE_PATH_STEPS = 4,
-    MOCE_PATH_RING = 5
+    MOCE_PATH_RING = 5,
+    MOCE_PATH_STREAM = 6
 } moce_path_t;
 
 /* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */

@@ -139,10 +139,15 @@ static moce_path_t pick_path(const void *x, int N, int HW, int C_in, int C_out, 
     const bool two = vec && ring_supported(N, HW, C_in, C_out, k, false);
     const bool ring = vec && ring_supported(N, HW, C_in, C_out, k, true);
     const bool fused = vec && fused_supported(N, HW, C_in, C_out, k);
+    const bool stream = vec && stream_supported(N, HW, C_in, C_out, k);
     switch (want) {
         case MOCE_PATH_AUTO:  // the fastest measured first
-            return two ? MOCE_PATH_TWO_PASS
-                       : pipe ? MOCE_PATH_PIPE : fused ? MOCE_PATH_FUSED : MOCE_PATH_STEPS;
+            return stream ? MOCE_PATH_STREAM
+                   : two  ? MOCE_PATH_TWO_PASS
+                   : pipe ? MOCE_PATH_PIPE
+                   : fused ? MOCE_PATH_FUSED
+                           : MOCE_PATH_STEPS;
+        case MOCE_PATH_STREAM: return stream ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_PIPE: return pipe ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_TWO_PASS: return two ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_FUSED: return fused ? want : MOCE_PATH_AUTO;
@@ -160,7 +165,7 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
                                 float tau_max, void *y, void *ws, size_t ws_bytes,
                                 moce_path_t path, moce_stream_t stream) {
     if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
-        !tau_ok(tau_min, tau_max) || path < MOCE_PATH_AUTO || path > MOCE_PATH_RING)
+        !tau_ok(tau_min, tau_max) || path < MOCE_PATH_AUTO || path > MOCE_PATH_STREAM)
         return MOCE_ERR_INVALID_VALUE;
     if (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
     const int HW = H * W;
@@ -191,6 +196,10 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
             return cuda_status(launch_fused(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
                                             resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
                                             yv, L, wsb, s));
+        case MOCE_PATH_STREAM:
+            return cuda_status(launch_stream(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
+                                             resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
+                                             yv, L, wsb, s));
         default: break;
     }
     float *z = reinterpret_cast<float *>(wsb + L.z);
@@ -225,13 +234,14 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
 int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                moce_dtype_t dtype, moce_layout_t layout, moce_path_t path) {
     if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
-        path < MOCE_PATH_AUTO || path > MOCE_PATH_RING)
+        path < MOCE_PATH_AUTO || path > MOCE_PATH_STREAM)
         return 0;
     if (N == 0 || H * W == 0) return 0;
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
     switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
         case MOCE_PATH_PIPE:
         case MOCE_PATH_FUSED:
+        case MOCE_PATH_STREAM:
         case MOCE_PATH_RING: return 1;
         case MOCE_PATH_TWO_PASS: return 2;  // pool+gate, then mix
         case MOCE_PATH_STEPS: return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
@@ -255,6 +265,7 @@ const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_i
         case MOCE_PATH_FUSED: return "moce_fused_kernel";
         case MOCE_PATH_STEPS: return "pool+gate+mix";
         case MOCE_PATH_RING: return "moce_ring_kernel";
+        case MOCE_PATH_STREAM: return "moce_stream_kernel";
         default: return nullptr;
     }
 }

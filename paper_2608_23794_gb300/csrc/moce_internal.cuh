@@ -61,12 +61,19 @@ struct WsLayout {
                           // softmax weight pairs in mixing-table order (two-pass path)
     size_t zacc = 0;      // [N][4][C] int64 fixed-point channel sums (two-pass path)
     size_t sync = 0;      // [2][N] uint32: tile arrivals, then the tag (epoch + 1) of the
-                          // forward that produced example n's weights (two-pass path)
+                          // forward that produced example n's weights (two-pass and stream paths)
+    size_t sblk = 0;      // [N] weight blocks of the stream path (stream_table_bytes(R) each)
     size_t total = 0;
     int pool_px = 0;
     int pool_tiles = 0;
     int gate_blocks = 0;
 };
+
+// Bytes of one example's weight block on the stream path: 16 floats per
+// expert plus 16 bytes per 8 experts (bank offset of the mixing groups).
+inline size_t stream_table_bytes(int R) {
+    return R <= 64 ? (size_t)64 * R + (size_t)16 * ((R + 7) / 8) : 0;
+}
 
 inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     WsLayout L;
@@ -87,6 +94,7 @@ inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     L.a = take((size_t)N * mx((size_t)R * k * 8, (size_t)4096));
     L.zacc = take((size_t)N * 4 * C * 8);
     L.sync = take((size_t)N * 8);
+    L.sblk = take((size_t)N * stream_table_bytes(R));
     L.total = off;
     return L;
 }
@@ -163,5 +171,13 @@ cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
                         bool fused, cudaStream_t s);
 
 bool ring_supported(int N, int HW, int C, int R, int k, bool fused);
+
+cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
+                          const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
+                          const float *W1, const float *b1, const float *w2, const float *b2,
+                          float tmin, float tmax, uint16_t *y, const WsLayout &L,
+                          unsigned char *ws, cudaStream_t s);
+
+bool stream_supported(int N, int HW, int C, int R, int k);
 
 }  // namespace moce

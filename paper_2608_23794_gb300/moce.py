@@ -213,7 +213,7 @@ def moce_gate(z: torch.Tensor, packed: PackedSupports, W1, b1, w2, b2, tau_min: 
 
 
 # moce_path_t: the kernel path of one forward (AUTO = the fastest that fits)
-PATHS = {"auto": 0, "pipe": 1, "two_pass": 2, "fused": 3, "steps": 4, "ring": 5}
+PATHS = {"auto": 0, "pipe": 1, "two_pass": 2, "fused": 3, "steps": 4, "ring": 5, "stream": 6}
 
 
 def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,

@@ -19,7 +19,7 @@ pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
 
 
-@pytest.mark.parametrize("path", ["pipe", "two_pass", "ring", "fused"])
+@pytest.mark.parametrize("path", ["stream", "pipe", "two_pass", "ring", "fused"])
 def test_bounded_wait_reports_timeout_and_recovers(path):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
