@@ -1,48 +1,55 @@
-// Single-pass streaming forward of a MoCE layer (Sec. 3.3-3.4) for NHWC bf16
-// layers with 64 <= C_in <= 256, C_in % 64 == 0, C_out <= 64, k <= 16 and at
-// most 255 tiles of 64 positions per example: x is read from HBM once.
+// Streaming forward of a MoCE layer (Sec. 3.3-3.4) for NHWC bf16 layers with
+// 64 <= C_in <= 256, C_in % 64 == 0, C_out <= 64, k <= 16 and at most 255
+// tiles of 64 positions per example, in one cooperative launch: x crosses
+// HBM once.
 //
 // Every expert's temperature needs the whole-image pool of its example
 // (Sec. 3.3, Eq. (tau)), so no position can be mixed before its example has
-// been pooled. Here a tile stays in shared memory from the moment it is
-// pooled until its example's gate has run, and is mixed from there.
+// been pooled. Each tile is therefore read twice through the GPU but once
+// from HBM: a pool stream reads it from HBM a few items ahead of the mix
+// stream, adds its channel sums to the example's accumulator words and lets
+// the slot go at once; the mix stream reads it again, from L2, once the
+// example's gate has (usually long) run. The streams wait on each other
+// only through two counters: the pool stream runs at most `lead` items ahead
+// of the mix stream's loads, and the mix stream loads only tiles the pool
+// stream has read. The latency from a tile's pooling to its example's
+// weights thus stalls no shared-memory slot.
 //
 // Work: tiles of 64 positions of one example (tile t of example n is item
-// it = n T + t, T = ceil(HW / 64)); CTA b of G (one per SM, cooperative
-// launch) takes items b, b + G, ... through a ring of D shared-memory slots.
-// Roles (640 threads):
-//   producer (warp 16)   : one TMA tensor load per 64-channel group of the
-//                          tile ([64 positions][64 channels], 128-byte
-//                          swizzle) into slot j mod D;
-//   transpose (0-3)      : warp g owns channel group g of the slot and, on
-//                          its own (no barrier with the other warps): reads
-//                          it with ldmatrix.trans, adds the tile's channel
-//                          sums (the pool, Sec. 3.3), writes the words back
-//                          in place as channel-major rows (row c = the
+// it = n T + t, T = ceil(HW / 64)). Stream CTA b of Gs takes items b,
+// b + Gs, ... in both streams; the other Gg CTAs (a few SMs) run the gates:
+// on a stream SM a gate would share issue slots and shared memory with the
+// mixing and come late. Roles of a stream CTA (640 threads):
+//   pool (warps 0-3)     : warp g reads channel group g of the pool slot
+//                          (ldmatrix.trans of the TMA's 128-byte swizzled
+//                          [64 positions][64 channels] block) and adds the
+//                          tile's channel sums (the pool, Sec. 3.3);
+//   transpose (4-7)      : warp g transposes channel group g of the mix slot
+//                          in place into channel-major rows (row c = the
 //                          tile's 64 positions of channel c, bf16 pairs) and
-//                          signals the slot;
-//   publish (18)         : adds the tile's channel sums to the example's
-//                          accumulator words by one bulk reduction;
-//   residual (19)        : sums the unselected channels of every position
-//                          (Eq. (res));
-//   gate (4-7)           : for every example whose last tile this CTA
-//                          holds, wait (bounded) until every accumulator
-//                          word of the example counts all T tiles, decode z,
-//                          run the gate of every expert (Eq. (tau)) and the
-//                          softmax weights (Eq. (weights)), publish them with
-//                          a tag. These warps wait for nothing else (no slot,
-//                          no other gate), so no chain of waits passes
-//                          through a gate;
-//   mix (8-15)           : each 8-lane group owns one expert pair with their
+//                          sums the group's unselected channels at every
+//                          position (Eq. (res));
+//   mix (8-15)           : each 8-lane group owns one expert pair, with their
 //                          row offsets and weights in registers; a lane reads
 //                          one 16-byte chunk (8 positions) of a support row
-//                          and adds it with fma.rn.f32x2 (Eq. (expert)); y
-//                          with the residual column is staged in shared
-//                          memory; the mix warps synchronise only through
-//                          mbarriers, never with a CTA barrier;
-//   table + store (17)   : brings the weights of item j's example (waiting,
-//                          bounded, for its tag) into one of two tables;
-//                          each staged y tile leaves by one bulk copy.
+//                          and adds it with fma.rn.f32x2 (Eq. (expert)); the
+//                          y tile with the residual column is staged in
+//                          shared memory;
+//   pool producer (16), mix producer (17): one 32 KB TMA tensor load per tile
+//                          (the pool stream's with an L2 evict_last policy and
+//                          an L2 prefetch a few items ahead, the mix stream's
+//                          evict_first); the mix producer also brings the
+//                          weights of each item's example (waiting, bounded,
+//                          for the tag its gate publishes) into one of two
+//                          tables by one bulk copy;
+//   store (18)           : each staged y tile (two staging buffers) leaves by
+//                          one bulk copy;
+//   publish (19)         : the channel sums go to the example's accumulator
+//                          words by one bulk reduction.
+// A gate CTA takes the examples g, g + Gg, ...: it waits (bounded) until
+// every accumulator word of the example counts all T tiles, decodes z, runs
+// the gate of every expert (Eq. (tau)) and the softmax weights
+// (Eq. (weights)), and publishes them with a tag.
 // Accumulator word of (example, channel): bits 56-63 count the tiles added,
 // bits 48-55 the tiles whose sum was kept as a tagged fp32 word instead,
 // bits 0-47 the sum of 2^39 + round(2^20 s) over the other tiles (s = the
@@ -60,41 +67,47 @@
 
 #include "moce_device.cuh"
 
+#ifndef MOCE_STREAM_LEAD
+#define MOCE_STREAM_LEAD 12
+#endif
+#ifndef MOCE_STREAM_DP
+#define MOCE_STREAM_DP 2
+#endif
+#ifndef MOCE_STREAM_PF
+#define MOCE_STREAM_PF 1
+#endif
+
 namespace moce {
 namespace {
 
 constexpr int kTP = 64;             // positions per tile
 constexpr int kThreads_ = 640;
-// Warps are ordered by how short their critical path is: the transpose and
-// gate warps come first (the scheduler favours older warps when several are
-// ready, and the mix warps, with many independent loads in flight, are
-// nearly always ready), the mix warps after them.
-constexpr int kTr0 = 0;             // warps 0-3
-constexpr int kGate0 = 128;         // warps 4-7
+constexpr int kPool0 = 0;           // warps 0-3
+constexpr int kTr0 = 128;           // warps 4-7
 constexpr int kMix0 = 256;          // warps 8-15
 constexpr int kMixT = 256;
-constexpr int kProdW = 16;          // warp 17: y stores; 18: pool words; 19: residual
-constexpr int kStoreW = 17;
-constexpr int kPubW = 18;
-constexpr int kResW = 19;
-constexpr int kMaxD = 6;            // x slots at most
+constexpr int kPoolProdW = 16, kMixProdW = 17, kStoreW = 18;  // warp 19 publishes
+constexpr int kDP = MOCE_STREAM_DP; // pool slots
+constexpr int kMaxDM = 6;           // mix slots at most
 constexpr int kNT = 2;              // weight tables
 constexpr int kKMax = 16;
 constexpr int kRMax = 64;
 constexpr int kMaxT = 255;          // tiles per example (8-bit count field)
-constexpr int kBarGate = 3;
-// mbarriers: raw (TMA landed), staged (transposed), empty (mixed), tready /
-// tfree (gate -> mix tables), ydone / yfree (mix -> store staging buffers)
-constexpr int kMbRaw = 0, kMbStaged = kMaxD, kMbEmpty = 2 * kMaxD, kMbTReady = 3 * kMaxD,
-              kMbTFree = 3 * kMaxD + kNT, kMbYDone = 3 * kMaxD + 2 * kNT,
-              kMbYFree = 3 * kMaxD + 2 * kNT + 1, kMbPooled = 3 * kMaxD + 2 * kNT + 2,
-              kMbPFree = 3 * kMaxD + 2 * kNT + 4, kMbResDone = 3 * kMaxD + 2 * kNT + 6,
-              kMbCount = 4 * kMaxD + 2 * kNT + 6;
-// registers: 96 per thread at launch; mix 136, transpose 104, gate 56, the rest 48
-// (setmaxnreg.inc waits for registers the other warpgroups release: the
-// shares must add up to no more than the launch allocation)
-constexpr int kRegLaunch = 96, kRegMix = 136, kRegTr = 104, kRegGate = 56, kRegMisc = 48;
-static_assert(2 * 128 * kRegMix + 128 * kRegTr + 128 * kRegGate + 128 * kRegMisc <=
+constexpr int kBarPool = 1;
+static_assert(kDP >= 2 && kDP <= 4, "pool slots");
+// mbarriers: praw / pfree (pool ring), mraw / staged / empty (mix ring),
+// tready / tfree (tables), ydone / yfree (y staging buffers), pooled / psfree
+// (channel-sum buffers)
+constexpr int kNY = 2;              // y staging buffers
+constexpr int kMbPRaw = 0, kMbPFree = kDP, kMbMRaw = 2 * kDP, kMbStaged = 2 * kDP + kMaxDM,
+              kMbEmpty = 2 * kDP + 2 * kMaxDM, kMbTReady = 2 * kDP + 3 * kMaxDM,
+              kMbTFree = kMbTReady + kNT, kMbYDone = kMbTFree + kNT, kMbYFree = kMbYDone + kNY,
+              kMbPooled = kMbYFree + kNY, kMbPsFree = kMbPooled + 2, kMbCount = kMbPsFree + 2;
+// registers: 96 per thread at launch; mix 136, transpose 96, pool 64 and
+// warps 16-19 48 (setmaxnreg.inc waits for registers the other warpgroups
+// release: the shares must add up to no more than the launch allocation)
+constexpr int kRegLaunch = 96, kRegMix = 136, kRegTr = 96, kRegPool = 64, kRegMisc = 48;
+static_assert(2 * 128 * kRegMix + 128 * kRegTr + 128 * kRegPool + 128 * kRegMisc <=
                   kThreads_ * kRegLaunch,
               "register split exceeds the launch allocation");
 
@@ -121,7 +134,7 @@ __device__ __forceinline__ float unfix20(long long fx) {
 
 struct StreamParams {
     uint16_t *y;
-    int N, HW, C, R, k, nU, T, nreg, G, D;
+    int N, HW, C, R, k, nU, T, nreg, Gs, Gg, DM, lead, PF;
     uint32_t items;
     const int32_t *pidx;
     const float *plog;
@@ -136,8 +149,11 @@ struct StreamParams {
     float *z, *tau;             // [N][C], [N][R]
     uint32_t tb_bytes;          // bytes of one weight table
     uint32_t ysb;               // bytes of one y staging buffer
-    uint32_t off_x, off_tab, off_ys, off_res, off_U, off_zs, off_w1t, off_b1, off_w2, off_psum,
-        off_pword, off_bar;
+    // stream CTAs
+    uint32_t off_pool, off_mix, off_tab, off_ys, off_res, off_U, off_Ur, off_psum, off_pword,
+        off_ctr, off_bar;
+    // gate CTAs
+    uint32_t g_zs, g_w1t, g_b1, g_w2, g_idx, g_dl;
     uint32_t smem_bytes;
 };
 
@@ -152,12 +168,24 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes)
                  : "memory");
 }
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm, int x, int y,
-                                            uint32_t mbar, uint64_t policy) {
+// Tile t of example n: the box {64 channels, 64 positions, 1, all channel
+// groups} of the four-dimensional view of x (see launch_stream) at position
+// 64 t of example n; positions past the example's last read as zeros.
+__device__ __forceinline__ void tma_load_tile(uint32_t dst, const CUtensorMap *tm, int t, int n,
+                                              uint32_t mbar, uint64_t policy) {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(mbar), "l"(policy)
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(0), "r"(kTP * t), "r"(n), "r"(0), "r"(mbar),
+        "l"(policy)
+        : "memory");
+}
+// Untiled bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes,
+                                          uint32_t mbar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(mbar)
         : "memory");
 }
 __device__ __forceinline__ void ldsm_x4_t(uint32_t a, uint32_t (&r)[4]) {
@@ -182,13 +210,16 @@ __device__ __forceinline__ uint4 lds128a(uint32_t a) {
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
 __device__ __forceinline__ void bulk_store(void *dst, uint32_t src, uint32_t bytes) {
     asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
                  "r"(src), "r"(bytes)
                  : "memory");
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    bulk_commit();
 }
-// Bulk stores of this thread still reading shared memory: at most N groups.
+// Bulk operations of this thread still reading shared memory: at most N groups.
 template <int N> __device__ __forceinline__ void bulk_wait_read() {
     asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
 }
@@ -198,9 +229,11 @@ __device__ __forceinline__ void bulk_wait_all() {
 __device__ __forceinline__ void fence_mbar_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
-// acc + lo, then + hi, for the two bf16 of a word (exact widening, fp32 add)
+// acc + lo, then + hi, for the two bf16 of a word (exact widening, fp32 add);
+// volatile, so that the adds keep their place between the ldmatrix loads
+// (hoisting all loads first would need more registers than the pool has)
 __device__ __forceinline__ float add_bf16x2(float acc, uint32_t w) {
-    asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\t"
+    asm volatile("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\t"
         "add.rn.f32.bf16 %0, lo, %0;\n\tadd.rn.f32.bf16 %0, hi, %0;\n\t}"
         : "+f"(acc)
         : "r"(w));
@@ -221,7 +254,26 @@ __device__ __forceinline__ void bulk_reduce_add_u64(void *dst, uint32_t src, uin
         "cp.reduce.async.bulk.global.shared::cta.bulk_group.add.u64 [%0], [%1], %2;" ::"l"(dst),
         "r"(src), "r"(bytes)
         : "memory");
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    bulk_commit();
+}
+// The two stream counters live in shared memory; the producers poll them.
+__device__ __forceinline__ uint32_t ld_ctr(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_ctr(uint32_t a, uint32_t v) {
+    asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+// Bounded wait until the counter at a exceeds v.
+__device__ bool wait_ctr(uint32_t a, uint32_t v, uint32_t *ctrl, uint32_t item) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+        if (ld_ctr(a) > v) return true;
+        if ((i & 15u) == 15u && ld_relaxed(ctrl + kCtrlError) != 0u) return false;
+        __nanosleep(i < 64 ? 20 : 200);
+    }
+    report_timeout(ctrl, item);
+    return false;
 }
 
 struct Item {
@@ -230,7 +282,7 @@ struct Item {
 };
 __device__ __forceinline__ Item item_of(const StreamParams &P, int j) {
     Item r;
-    r.it = (uint32_t)blockIdx.x + (uint32_t)j * (uint32_t)P.G;
+    r.it = (uint32_t)blockIdx.x + (uint32_t)j * (uint32_t)P.Gs;
     r.n = (int)(r.it / (uint32_t)P.T);
     r.t = (int)(r.it - (uint32_t)r.n * (uint32_t)P.T);
     r.valid = min(kTP, P.HW - r.t * kTP);
@@ -238,118 +290,166 @@ __device__ __forceinline__ Item item_of(const StreamParams &P, int j) {
 }
 __device__ __forceinline__ int items_of_cta(const StreamParams &P) {
     const uint32_t b = blockIdx.x;
-    return b < P.items ? (int)((P.items - 1u - b) / (uint32_t)P.G) + 1 : 0;
+    return b < P.items ? (int)((P.items - 1u - b) / (uint32_t)P.Gs) + 1 : 0;
 }
-__device__ __forceinline__ float *res_of(const StreamParams &P, unsigned char *sm, int s) {
-    return reinterpret_cast<float *>(sm + P.off_res) + s * kTP;
+// residual partial of channel group g for mix slot s: [64 positions] fp32
+__device__ __forceinline__ float *res_part(const StreamParams &P, unsigned char *sm, int s, int g) {
+    return reinterpret_cast<float *>(sm + P.off_res) + (s * 4 + g) * kTP;
+}
+// counter 0: items the pool stream has pooled; counter 1: items the mix
+// stream has loaded
+__device__ __forceinline__ uint32_t ctr_addr(const StreamParams &P, unsigned char *sm, int i) {
+    return smem_u32(sm + P.off_ctr) + 4u * (uint32_t)i;
 }
 
 // ================================================================ roles
 
-// Producer: one TMA tensor load per 64-channel group of each tile.
-__device__ void role_producer(const StreamParams &P, const CUtensorMap *tm, unsigned char *sm) {
+// Pool producer: the pool stream's TMA loads (evict_last: the mix stream
+// reads the same lines again from L2), at most `lead` items ahead of the mix
+// stream's loads.
+__device__ void role_pool_producer(const StreamParams &P, const CUtensorMap *tm,
+                                   unsigned char *sm) {
     if ((threadIdx.x & 31) != 0) return;
     const uint32_t bar = smem_u32(sm + P.off_bar);
-    const uint32_t xs0 = smem_u32(sm + P.off_x);
+    const uint32_t xs0 = smem_u32(sm + P.off_pool);
     const uint32_t sb = (uint32_t)P.C * kTP * 2u;
     uint64_t pol;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
     const int nj = items_of_cta(P);
+    // L2 prefetch of item j + PF with the load of item j: HBM gets PF tiles in
+    // flight without holding shared memory, and the loads hit L2
+    auto prefetch = [&](int j) {
+        const Item I = item_of(P, j);
+        asm volatile(
+            "cp.async.bulk.prefetch.tensor.4d.L2.global.tile.L2::cache_hint"
+            " [%0, {%1, %2, %3, %4}], %5;"
+            ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(0), "r"(kTP * I.t), "r"(I.n), "r"(0),
+            "l"(pol)
+            : "memory");
+    };
+    for (int j = 0; j < min(P.PF, nj); ++j) prefetch(j);
     int issued = 0;
     for (int j = 0; j < nj; ++j) {
-        const int s = j % P.D;
-        if (j >= P.D &&
-            !mbar_wait(bar + 8u * (kMbEmpty + s), (uint32_t)((j / P.D) - 1) & 1u, P.ctrl, 0u))
+        const int s = j % kDP;
+        if (j >= kDP &&
+            !mbar_wait(bar + 8u * (kMbPFree + s), (uint32_t)((j / kDP) - 1) & 1u, P.ctrl, 0u))
+            break;
+        if (j >= P.lead && !wait_ctr(ctr_addr(P, sm, 1), (uint32_t)(j - P.lead), P.ctrl, 0u))
             break;
         const Item I = item_of(P, j);
-        const int row = I.n * P.HW + I.t * kTP;
-        const uint32_t full = bar + 8u * (kMbRaw + s);
-        mbar_expect_tx(full, (uint32_t)P.nreg * 8192u);
-        for (int g = 0; g < P.nreg; ++g)
-            tma_load_2d(xs0 + (uint32_t)s * sb + 8192u * (uint32_t)g, tm, 64 * g, row, full, pol);
+        if (j + P.PF < nj) prefetch(j + P.PF);
+        const uint32_t full = bar + 8u * (kMbPRaw + s);
+        mbar_expect_tx(full, sb);
+        tma_load_tile(xs0 + (uint32_t)s * sb, tm, I.t, I.n, full, pol);
         ++issued;
     }
     // no copy may still be writing shared memory when the CTA exits
-    for (int j = issued > P.D ? issued - P.D : 0; j < issued; ++j)
-        mbar_wait(bar + 8u * (kMbRaw + j % P.D), (uint32_t)(j / P.D) & 1u, P.ctrl, 0u);
+    for (int j = issued > kDP ? issued - kDP : 0; j < issued; ++j)
+        mbar_wait(bar + 8u * (kMbPRaw + j % kDP), (uint32_t)(j / kDP) & 1u, P.ctrl, 0u);
 }
 
-// Transpose + pool, warp g on channel group g alone. Region g of the slot
-// (8 KB) holds [64 positions][64 channels] as the TMA wrote it (128-byte
-// swizzle: 16-byte chunk c of row p at chunk c ^ (p & 7)). ldmatrix.trans of
-// 8x8 blocks gives lane l (cl = l / 4, q = l mod 4) the words
-// {x[p][c], x[p + 1][c]} for channel c = 8 jj + cl of the region and
-// positions p = 32 h + 8 m + 2 q (m = 0..3 over the four matrices). The lane
-// adds them to its channel sums (the pool, Sec. 3.3) and stores its four
-// words as one 16-byte chunk at logical chunk 4 h + q of row c (physical
-// chunk (4 h + q) ^ (4 (c & 1))): row c then holds the tile's 64 positions
-// of channel c, word 16 h + 4 q + m holding positions 2 (16 h + 4 m + q) and
-// the next. The channel sums go to the publish warp, the slot to the
-// residual and mix warps: nothing else stands on this warp's path.
-__device__ void role_transpose(const StreamParams &P, unsigned char *sm) {
-    const int tt = threadIdx.x - kTr0;  // 0..127
+// Mix producer: the mix stream's TMA loads (evict_first: the lines are dead
+// after this read), each once the pool stream has read the tile, so that it
+// comes from L2; then the weights of the item's example, once its gate has
+// published them (bounded wait on the tag), into table j mod kNT by one bulk
+// copy, once the mix warps have read that table's item j - kNT.
+__device__ void role_mix_producer(const StreamParams &P, const CUtensorMap *tm,
+                                  unsigned char *sm, uint32_t tag) {
+    if ((threadIdx.x & 31) != 0) return;
+    const uint32_t bar = smem_u32(sm + P.off_bar);
+    const uint32_t xs0 = smem_u32(sm + P.off_mix);
+    const uint32_t tb0 = smem_u32(sm + P.off_tab);
+    const uint32_t sb = (uint32_t)P.C * kTP * 2u;
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    const int nj = items_of_cta(P);
+    int issued = 0, tabs = 0;
+    for (int j = 0; j < nj; ++j) {
+        const Item I = item_of(P, j);
+        const int s = j % P.DM, q = j % kNT;
+        if (j >= P.DM && !mbar_wait(bar + 8u * (kMbEmpty + s), (uint32_t)((j / P.DM) - 1) & 1u,
+                                    P.ctrl, I.it))
+            break;
+        if (!wait_ctr(ctr_addr(P, sm, 0), (uint32_t)j, P.ctrl, I.it)) break;
+        const uint32_t full = bar + 8u * (kMbMRaw + s);
+        mbar_expect_tx(full, sb);
+        tma_load_tile(xs0 + (uint32_t)s * sb, tm, I.t, I.n, full, pol);
+        ++issued;
+        st_ctr(ctr_addr(P, sm, 1), (uint32_t)issued);
+        if (j >= kNT && !mbar_wait(bar + 8u * (kMbTFree + q), (uint32_t)((j / kNT) - 1) & 1u,
+                                   P.ctrl, I.it))
+            break;
+        bool ok = false;
+        for (uint32_t i = 0; i < kSpinLimit; ++i) {
+            if (ld_acquire(P.flag + I.n) == tag) { ok = true; break; }
+            if ((i & 15u) == 15u && ld_relaxed(P.ctrl + kCtrlError) != 0u) break;
+            __nanosleep(i < 64 ? 20 : 100);
+        }
+        if (!ok) {
+            if (ld_relaxed(P.ctrl + kCtrlError) == 0u) report_timeout(P.ctrl, I.it);
+            break;
+        }
+        // the gate's stores (generic proxy, seen through the acquire) before
+        // the bulk copy's reads (async proxy)
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+        const uint32_t tfull = bar + 8u * (kMbTReady + q);
+        mbar_expect_tx(tfull, P.tb_bytes);
+        bulk_load(tb0 + (uint32_t)q * P.tb_bytes, P.wblk + (size_t)I.n * (P.tb_bytes >> 2),
+                  P.tb_bytes, tfull);
+        ++tabs;
+    }
+    // no copy may still be writing shared memory when the CTA exits
+    for (int j = issued > P.DM ? issued - P.DM : 0; j < issued; ++j)
+        mbar_wait(bar + 8u * (kMbMRaw + j % P.DM), (uint32_t)(j / P.DM) & 1u, P.ctrl, 0u);
+    for (int j = tabs > kNT ? tabs - kNT : 0; j < tabs; ++j)
+        mbar_wait(bar + 8u * (kMbTReady + j % kNT), (uint32_t)(j / kNT) & 1u, P.ctrl, 0u);
+}
+
+// Pool, warp g on channel group g. Region g of the pool slot (8 KB) holds
+// [64 positions][64 channels] as the TMA wrote it (128-byte swizzle: 16-byte
+// chunk c of row p at chunk c ^ (p & 7)); ldmatrix.trans of 8x8 blocks gives
+// lane l (cl = l / 4, q = l mod 4) the words {x[p][c], x[p + 1][c]} for
+// channel c = 8 jj + cl of the region and positions p = 32 h + 8 m + 2 q.
+// The lane adds them per channel; the four lanes of a channel (q) are added
+// in a fixed order and the tile's channel sums go to sum buffer j mod 2 for
+// the publish warp. Once every warp has read the slot it goes back to the
+// producer, and the item counts as loaded for the mix stream.
+__device__ void role_pool(const StreamParams &P, unsigned char *sm) {
+    const int tt = threadIdx.x - kPool0;  // 0..127
     const int g = tt >> 5, lane = tt & 31;
     const int q = lane & 3, cl = lane >> 2;
     const uint32_t bar = smem_u32(sm + P.off_bar);
-    const uint32_t xs0 = smem_u32(sm + P.off_x);
+    const uint32_t xs0 = smem_u32(sm + P.off_pool);
     const uint32_t sb = (uint32_t)P.C * kTP * 2u;
     const bool own = g < P.nreg;
     const int nj = items_of_cta(P);
     for (int j = 0; j < nj; ++j) {
         const Item I = item_of(P, j);
-        const int s = j % P.D, pb = j & 1;
-        bool ok = mbar_wait(bar + 8u * (kMbRaw + s), (uint32_t)(j / P.D) & 1u, P.ctrl, I.it);
-        // the publish warp has read this sum buffer (item j - 2)
-        ok = ok && (j < 2 || mbar_wait(bar + 8u * (kMbPFree + pb), (uint32_t)((j >> 1) - 1) & 1u,
+        const int s = j % kDP, pb = j & 1;
+        bool ok = mbar_wait(bar + 8u * (kMbPRaw + s), (uint32_t)(j / kDP) & 1u, P.ctrl, I.it);
+        // the publish warp has read sum buffer pb (item j - 2)
+        ok = ok && (j < 2 || mbar_wait(bar + 8u * (kMbPsFree + pb), (uint32_t)((j >> 1) - 1) & 1u,
                                        P.ctrl, I.it));
-        if (!__all_sync(0xffffffffu, ok)) break;  // warp-uniform exit
-        if (own) {
-            const uint32_t rb = xs0 + (uint32_t)s * sb + 8192u * (uint32_t)g;
-            uint32_t r[16][4];
+        if (ok && own) {
+            float pacc[8];
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+            for (int jj = 0; jj < 8; ++jj) pacc[jj] = 0.f;
+            const uint32_t rb = xs0 + (uint32_t)s * sb + 8192u * (uint32_t)g;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t r[8][4];
 #pragma unroll
                 for (int jj = 0; jj < 8; ++jj)
                     ldsm_x4_t(rb + (uint32_t)(32 * h + lane) * 128u +
                                   ((uint32_t)(jj ^ (lane & 7)) << 4),
-                              r[8 * h + jj]);
-            float pacc[8];
+                              r[jj]);
+                // positions past the example are zeros (the TMA fill)
 #pragma unroll
-            for (int jj = 0; jj < 8; ++jj) pacc[jj] = 0.f;
-            // the tile's channel sums (positions beyond the example excluded)
-            if (I.valid == kTP) {
+                for (int m = 0; m < 4; ++m)
 #pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int m = 0; m < 4; ++m)
-#pragma unroll
-                        for (int jj = 0; jj < 8; ++jj)
-                            pacc[jj] = add_bf16x2(pacc[jj], r[8 * h + jj][m]);
-            } else {
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int m = 0; m < 4; ++m) {
-                        // keep position p (low half) and p + 1 (high half) when in the example
-                        const int p = 32 * h + 8 * m + 2 * q;
-                        const uint32_t keep = (p < I.valid ? 0x0000ffffu : 0u) |
-                                              (p + 1 < I.valid ? 0xffff0000u : 0u);
-#pragma unroll
-                        for (int jj = 0; jj < 8; ++jj)
-                            pacc[jj] = add_bf16x2(pacc[jj], r[8 * h + jj][m] & keep);
-                    }
+                    for (int jj = 0; jj < 8; ++jj) pacc[jj] = add_bf16x2(pacc[jj], r[jj][m]);
             }
-            __syncwarp();
-#pragma unroll
-            for (int h = 0; h < 2; ++h)
-#pragma unroll
-                for (int jj = 0; jj < 8; ++jj) {
-                    const int c = 8 * jj + cl;
-                    sts128(rb + (uint32_t)c * 128u + ((uint32_t)((4 * h + q) ^ ((c & 1) << 2)) << 4),
-                           r[8 * h + jj]);
-                }
-            // sums over the four position subsets (lanes q = 0..3), in a fixed order
             float *ps = reinterpret_cast<float *>(sm + P.off_psum) + pb * P.C + 64 * g;
 #pragma unroll
             for (int jj = 0; jj < 8; ++jj) {
@@ -358,11 +458,12 @@ __device__ void role_transpose(const StreamParams &P, unsigned char *sm) {
                 v += __shfl_xor_sync(0xffffffffu, v, 2);
                 if ((jj & 3) == q) ps[8 * jj + cl] = v;
             }
-            __syncwarp();
         }
-        if (lane == 0) {
-            mbar_arrive(bar + 8u * (kMbStaged + s));
+        if (!bar_and(kBarPool, 128, ok)) break;  // every warp has read the slot
+        if (tt == 0) {
+            mbar_arrive(bar + 8u * (kMbPFree + s));
             mbar_arrive(bar + 8u * (kMbPooled + pb));
+            st_ctr(ctr_addr(P, sm, 0), (uint32_t)(j + 1));
         }
     }
 }
@@ -380,8 +481,8 @@ __device__ void role_publish(const StreamParams &P, unsigned char *sm) {
     for (int j = 0; j < nj; ++j) {
         const Item I = item_of(P, j);
         const int pb = j & 1;
-        if (!__all_sync(0xffffffffu, mbar_wait(bar + 8u * (kMbPooled + pb), (uint32_t)(j >> 1) & 1u,
-                                                P.ctrl, I.it)))
+        if (!__all_sync(0xffffffffu, mbar_wait(bar + 8u * (kMbPooled + pb),
+                                                (uint32_t)(j >> 1) & 1u, P.ctrl, I.it)))
             break;  // warp-uniform exit
         const float *ps = reinterpret_cast<const float *>(sm + P.off_psum) + pb * P.C;
         const uint32_t pw = smem_u32(sm + P.off_pword) + (uint32_t)pb * (uint32_t)P.C * 8u;
@@ -396,273 +497,282 @@ __device__ void role_publish(const StreamParams &P, unsigned char *sm) {
                 st_tagged(P.wide + ((size_t)I.n * P.T + I.t) * P.C + c, v, tag);
                 add = kTileOne + kWideOne;
             }
-            asm volatile("st.shared.u64 [%0], %1;" ::"r"(pw + 8u * (uint32_t)c), "l"(add) : "memory");
+            asm volatile("st.shared.u64 [%0], %1;" ::"r"(pw + 8u * (uint32_t)c), "l"(add)
+                         : "memory");
         }
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-            mbar_arrive(bar + 8u * (kMbPFree + pb));
+            mbar_arrive(bar + 8u * (kMbPsFree + pb));
             if (I.it + 1u != drop)  // fault injection: never counted
                 bulk_reduce_add_u64(zb + (size_t)I.n * P.C, pw, (uint32_t)P.C * 8u);
+            else
+                bulk_commit();  // an empty group keeps one group per item
         }
     }
     if (lane == 0) bulk_wait_all();  // the last reductions are complete
 }
 
-// Residual expert (Eq. (res)): the mean of the unselected channels at each
-// position of the transposed tile; lane (part = lane / 8, chunk jc = lane
-// mod 8) adds U entries part, part + 4, ... over its chunk's 8 positions,
-// then the four parts are added in a fixed order.
-__device__ void role_residual(const StreamParams &P, unsigned char *sm) {
-    const int lane = threadIdx.x & 31;
-    const int jc = lane & 7, part = lane >> 3;
+// Transpose, warp g on channel group g of the mix slot, in place: the lane's
+// four ldmatrix words (positions 32 h + 8 m + 2 q, m = 0..3, of channel
+// c = 8 jj + cl) go as one 16-byte chunk to logical chunk 4 h + q of row c
+// (physical chunk (4 h + q) ^ (4 (c & 1))): row c then holds the tile's 64
+// positions of channel c, word 16 h + 4 q + m holding positions
+// 2 (16 h + 4 m + q) and the next. Then the residual expert (Eq. (res)) over
+// the group's unselected channels: lane (part = lane / 8, chunk jc = lane
+// mod 8) adds the group's entries of U part, part + 4, ... over its chunk's
+// 8 positions, the four parts in a fixed order.
+__device__ void role_transpose(const StreamParams &P, unsigned char *sm) {
+    const int tt = threadIdx.x - kTr0;  // 0..127
+    const int g = tt >> 5, lane = tt & 31;
+    const int q = lane & 3, cl = lane >> 2;
     const uint32_t bar = smem_u32(sm + P.off_bar);
-    const uint32_t xs0 = smem_u32(sm + P.off_x);
+    const uint32_t xs0 = smem_u32(sm + P.off_mix);
     const uint32_t sb = (uint32_t)P.C * kTP * 2u;
+    const bool own = g < P.nreg;
+    // the entries of U in channel group g, in U's order (ballot compaction)
     const uint16_t *Us = reinterpret_cast<const uint16_t *>(sm + P.off_U);
+    uint16_t *Ur = reinterpret_cast<uint16_t *>(sm + P.off_Ur) + g * P.C;
+    int nr = 0;
+    for (int u0 = 0; u0 < P.nU; u0 += 32) {
+        const int u = u0 + lane;
+        const int c = u < P.nU ? (int)Us[u] : -1;
+        const bool mine = own && (c >> 6) == g;
+        const uint32_t bal = __ballot_sync(0xffffffffu, mine);
+        if (mine) Ur[nr + __popc(bal & ((1u << lane) - 1u))] = (uint16_t)c;
+        nr += __popc(bal);
+    }
+    __syncwarp();
     const int nj = items_of_cta(P);
     for (int j = 0; j < nj; ++j) {
         const Item I = item_of(P, j);
-        const int s = j % P.D;
-        if (!__all_sync(0xffffffffu, mbar_wait(bar + 8u * (kMbStaged + s), (uint32_t)(j / P.D) & 1u,
-                                                P.ctrl, I.it)))
+        const int s = j % P.DM;
+        if (!__all_sync(0xffffffffu,
+                        mbar_wait(bar + 8u * (kMbMRaw + s), (uint32_t)(j / P.DM) & 1u, P.ctrl, I.it)))
             break;  // warp-uniform exit
         const uint32_t xs = xs0 + (uint32_t)s * sb;
-        float2 ra[4];
+        if (own) {
+            const uint32_t rb = xs + 8192u * (uint32_t)g;
+            uint32_t r[16][4];
 #pragma unroll
-        for (int m = 0; m < 4; ++m) ra[m] = make_float2(0.f, 0.f);
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj)
+                    ldsm_x4_t(rb + (uint32_t)(32 * h + lane) * 128u +
+                                  ((uint32_t)(jj ^ (lane & 7)) << 4),
+                              r[8 * h + jj]);
+            __syncwarp();
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj) {
+                    const int c = 8 * jj + cl;
+                    sts128(rb + (uint32_t)c * 128u + ((uint32_t)((4 * h + q) ^ ((c & 1) << 2)) << 4),
+                           r[8 * h + jj]);
+                }
+            __syncwarp();
+            const int jc = lane & 7, part = lane >> 3;
+            float2 ra[4];
+#pragma unroll
+            for (int m = 0; m < 4; ++m) ra[m] = make_float2(0.f, 0.f);
 #pragma unroll 2
-        for (int u = part; u < P.nU; u += 4) {
-            const int c = Us[u];
-            const uint4 v = lds128a(xs + (uint32_t)c * 128u + ((uint32_t)(jc ^ ((c & 1) << 2)) << 4));
-            ra[0] = add_bf16_pair(ra[0], v.x);
-            ra[1] = add_bf16_pair(ra[1], v.y);
-            ra[2] = add_bf16_pair(ra[2], v.z);
-            ra[3] = add_bf16_pair(ra[3], v.w);
-        }
-#pragma unroll
-        for (int m = 0; m < 4; ++m) {
-#pragma unroll
-            for (int o = 8; o <= 16; o <<= 1) {
-                ra[m].x += __shfl_xor_sync(0xffffffffu, ra[m].x, o);
-                ra[m].y += __shfl_xor_sync(0xffffffffu, ra[m].y, o);
+            for (int u = part; u < nr; u += 4) {
+                const int c = Ur[u];
+                const uint4 v =
+                    lds128a(xs + (uint32_t)c * 128u + ((uint32_t)(jc ^ ((c & 1) << 2)) << 4));
+                ra[0] = add_bf16_pair(ra[0], v.x);
+                ra[1] = add_bf16_pair(ra[1], v.y);
+                ra[2] = add_bf16_pair(ra[2], v.z);
+                ra[3] = add_bf16_pair(ra[3], v.w);
             }
-        }
-        if (lane < 8) {
-            // positions 32 (jc / 4) + 8 m + 2 (jc mod 4) + {0, 1}
-            float *rp = res_of(P, sm, s);
 #pragma unroll
             for (int m = 0; m < 4; ++m) {
-                const int p = 32 * (jc >> 2) + 8 * m + 2 * (jc & 3);
-                rp[p] = ra[m].x * P.inv_nU;
-                rp[p + 1] = ra[m].y * P.inv_nU;
+#pragma unroll
+                for (int o = 8; o <= 16; o <<= 1) {
+                    ra[m].x += __shfl_xor_sync(0xffffffffu, ra[m].x, o);
+                    ra[m].y += __shfl_xor_sync(0xffffffffu, ra[m].y, o);
+                }
             }
+            if (lane < 8) {
+                // positions 32 (jc / 4) + 8 m + 2 (jc mod 4) + {0, 1}
+                float *rp = res_part(P, sm, s, g);
+#pragma unroll
+                for (int m = 0; m < 4; ++m) {
+                    const int p = 32 * (jc >> 2) + 8 * m + 2 * (jc & 3);
+                    rp[p] = ra[m].x;
+                    rp[p + 1] = ra[m].y;
+                }
+            }
+            __syncwarp();
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar + 8u * (kMbResDone + s));
+        if (lane == 0) mbar_arrive(bar + 8u * (kMbStaged + s));
     }
 }
 
-// Gate of every expert of example n (Eq. (tau)) and its softmax weights
-// (Eq. (weights)) into the example's weight block in global memory, by the
-// 128 threads of the gate role; thread (e = gt / 2, h = gt mod 2) holds
-// hidden units 8 h .. 8 h + 7 and support positions 8 h .. 8 h + 7 of expert
-// e. W1 is kept transposed and zero-padded to 16 x 16 (W1t[i][j] = W1[j][i]),
-// b1 and w2 zero-padded to 16, so padded units and positions contribute
-// nothing. z and tau of the example are written out as well.
+// Gate CTA: the examples n = g, g + Gg, ... (g = its index among the Gg gate
+// CTAs), in order. For each, thread c waits (bounded) until accumulator word
+// c of the example counts all T tiles and decodes z_c; then thread
+// 4 e + q runs hidden units 4 q .. 4 q + 3 of expert e's gate (Eq. (tau))
+// and its softmax weights 4 q .. 4 q + 3 (Eq. (weights)), the four threads
+// of an expert adding their partial sums in a fixed order; the weights go to
+// the example's weight block in global memory, published with a tag. W1 is
+// kept transposed and zero-padded to 16 x 16 (W1t[i][j] = W1[j][i]), b1 and w2
+// zero-padded to 16, and per expert its support channels and logit offsets
+// L_i - L_0 (L_0 the largest), so padded units and entries add nothing.
 template <int KT>
-__device__ bool gate_example(const StreamParams &P, unsigned char *sm, int n, uint32_t tag,
-                             uint32_t item) {
-    const int gt = threadIdx.x - kGate0;
-    float *zs = reinterpret_cast<float *>(sm + P.off_zs);
-    const float4 *W1t = reinterpret_cast<const float4 *>(sm + P.off_w1t);
-    const float *b1s = reinterpret_cast<const float *>(sm + P.off_b1);
-    const float *w2s = reinterpret_cast<const float *>(sm + P.off_w2);
-    constexpr int k = KT;
+__device__ void gate_cta(const StreamParams &P, unsigned char *sm, uint32_t tag) {
+    const int tid = threadIdx.x;
+    float *zs = reinterpret_cast<float *>(sm + P.g_zs);
+    const float4 *W1t = reinterpret_cast<const float4 *>(sm + P.g_w1t);
+    const float *b1s = reinterpret_cast<const float *>(sm + P.g_b1);
+    const float *w2s = reinterpret_cast<const float *>(sm + P.g_w2);
+    const uint16_t *gidx = reinterpret_cast<const uint16_t *>(sm + P.g_idx);
+    const float4 *gdl = reinterpret_cast<const float4 *>(sm + P.g_dl);
     const unsigned long long T = (unsigned long long)P.T;
-    const unsigned long long *zb = P.zacc + ((size_t)((tag - 1u) & 1u) * P.N + n) * P.C;
-    // z from the accumulator words, once each counts every tile (bounded)
-    bool ok = true;
-    for (int c = gt; c < P.C; c += 128) {
-        unsigned long long w = ld_relaxed64(zb + c);
-        for (uint32_t i = 0; (w >> 56) != T && i < kSpinLimit; ++i) {
-            if ((i & 15u) == 15u && ld_relaxed(P.ctrl + kCtrlError) != 0u) break;
-            __nanosleep(i < 64 ? 20 : 200);
-            w = ld_relaxed64(zb + c);
-        }
-        if ((w >> 56) != T) {
-            ok = false;
-            break;
-        }
-        const unsigned long long nw = (w >> 48) & 0xffull;
-        const long long fx =
-            (long long)(w & ((1ull << 48) - 1ull)) - (long long)((T - nw) * kFixBias);
-        float sum = unfix20(fx);
-        if (nw != 0ull) {
-            // the tagged fp32 sums of the wide tiles, in tile order, once each
-            // carries this forward's tag (bounded)
-            const unsigned long long *wp = P.wide + (size_t)n * P.T * P.C + c;
-            bool got = false;
-            for (uint32_t rep = 0; rep < kSpinLimit && !got; ++rep) {
-                float acc = 0.f;
-                unsigned long long seen = 0;
-                for (int t = 0; t < P.T; ++t) {
-                    const unsigned long long wv = ld_tagged(wp + (size_t)t * P.C);
-                    if (tag_ok(wv, tag)) {
-                        acc += tag_val(wv);
-                        ++seen;
+    const float b2 = __ldg(P.b2);
+    for (int n = (int)blockIdx.x - P.Gs; n < P.N; n += P.Gg) {
+        const uint32_t item = (uint32_t)n * (uint32_t)P.T + (uint32_t)P.T - 1u;
+        // z from the accumulator words, once each counts every tile (bounded)
+        bool ok = true;
+        if (tid < P.C) {
+            const int c = tid;
+            const unsigned long long *zb = P.zacc + ((size_t)((tag - 1u) & 1u) * P.N + n) * P.C;
+            unsigned long long w = ld_relaxed64(zb + c);
+            for (uint32_t i = 0; (w >> 56) != T && i < kSpinLimit; ++i) {
+                if ((i & 15u) == 15u && ld_relaxed(P.ctrl + kCtrlError) != 0u) break;
+                __nanosleep(i < 256 ? 20 : 100);
+                w = ld_relaxed64(zb + c);
+            }
+            ok = (w >> 56) == T;
+            float sum = 0.f;
+            if (ok) {
+                const unsigned long long nw = (w >> 48) & 0xffull;
+                const long long fx =
+                    (long long)(w & ((1ull << 48) - 1ull)) - (long long)((T - nw) * kFixBias);
+                sum = unfix20(fx);
+                if (nw != 0ull) {
+                    // the tagged fp32 sums of the wide tiles, in tile order, once
+                    // each carries this forward's tag (bounded)
+                    const unsigned long long *wp = P.wide + (size_t)n * P.T * P.C + c;
+                    bool got = false;
+                    for (uint32_t rep = 0; rep < kSpinLimit && !got; ++rep) {
+                        float acc = 0.f;
+                        unsigned long long seen = 0;
+                        for (int t = 0; t < P.T; ++t) {
+                            const unsigned long long wv = ld_tagged(wp + (size_t)t * P.C);
+                            if (tag_ok(wv, tag)) {
+                                acc += tag_val(wv);
+                                ++seen;
+                            }
+                        }
+                        if (seen == nw) {
+                            sum += acc;
+                            got = true;
+                        } else if (ld_relaxed(P.ctrl + kCtrlError) != 0u) {
+                            break;
+                        } else {
+                            __nanosleep(200);
+                        }
                     }
-                }
-                if (seen == nw) {
-                    sum += acc;
-                    got = true;
-                } else if (ld_relaxed(P.ctrl + kCtrlError) != 0u) {
-                    break;
-                } else {
-                    __nanosleep(200);
+                    ok = got;
                 }
             }
-            if (!got) {
-                ok = false;
-                break;
+            const float zv = sum * P.inv_HW;
+            zs[c] = zv;
+            P.z[(size_t)n * P.C + c] = zv;
+            if (!ok && ld_relaxed(P.ctrl + kCtrlError) == 0u) report_timeout(P.ctrl, item);
+        }
+        if (!__syncthreads_and(ok)) break;
+        // whole warps (the shuffles need every lane); only threads below 4 R write
+        if (tid < ((4 * P.R + 31) & ~31)) {
+            const int e = min(tid >> 2, P.R - 1), q = tid & 3;
+            const bool wr = tid < 4 * P.R;
+            // h_j = b1_j + sum_i W1[j][i] u_i, in input order, for j = 4 q .. 4 q + 3
+            float4 h = reinterpret_cast<const float4 *>(b1s)[q];
+#pragma unroll
+            for (int i = 0; i < KT; ++i) {
+                const float ui = zs[gidx[e * 16 + i]];
+                const float4 w = W1t[4 * i + q];
+                h.x = fmaf(w.x, ui, h.x);
+                h.y = fmaf(w.y, ui, h.y);
+                h.z = fmaf(w.z, ui, h.z);
+                h.w = fmaf(w.w, ui, h.w);
+            }
+            const float4 w2 = reinterpret_cast<const float4 *>(w2s)[q];
+            float g = w2.x * fmaxf(h.x, 0.f);
+            g = fmaf(w2.y, fmaxf(h.y, 0.f), g);
+            g = fmaf(w2.z, fmaxf(h.z, 0.f), g);
+            g = fmaf(w2.w, fmaxf(h.w, 0.f), g);
+            g += __shfl_xor_sync(0xffffffffu, g, 1);
+            g += __shfl_xor_sync(0xffffffffu, g, 2);
+            const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-(g + b2)));
+            // a_i = exp((L_i - L_0) / tau) / sum_j exp((L_j - L_0) / tau)
+            const float rt = 1.f / tau;
+            const float4 d = gdl[e * 4 + q];
+            float4 ex;
+            ex.x = 4 * q + 0 < KT ? expf(d.x * rt) : 0.f;
+            ex.y = 4 * q + 1 < KT ? expf(d.y * rt) : 0.f;
+            ex.z = 4 * q + 2 < KT ? expf(d.z * rt) : 0.f;
+            ex.w = 4 * q + 3 < KT ? expf(d.w * rt) : 0.f;
+            float S = (ex.x + ex.y) + (ex.z + ex.w);
+            S += __shfl_xor_sync(0xffffffffu, S, 1);
+            S += __shfl_xor_sync(0xffffffffu, S, 2);
+            const float inv = 1.f / S;
+            if (wr) {
+                reinterpret_cast<float4 *>(P.wblk + (size_t)n * (P.tb_bytes >> 2) + wofs(e))[q] =
+                    make_float4(ex.x * inv, ex.y * inv, ex.z * inv, ex.w * inv);
+                if (q == 0) P.tau[(size_t)n * P.R + e] = tau;
             }
         }
-        const float zv = sum * P.inv_HW;
-        zs[c] = zv;
-        P.z[(size_t)n * P.C + c] = zv;
-    }
-    if (!ok && ld_relaxed(P.ctrl + kCtrlError) == 0u) report_timeout(P.ctrl, item);
-    if (!bar_and(kBarGate, 128, ok)) return false;
-    const int e = gt >> 1, h = gt & 1;
-    const bool act = e < P.R;
-    const int ec = act ? e : 0;
-    const int32_t *pi = P.pidx + ec * k;
-    const float *pl = P.plog + ec * k;
-    float u[KT];
-#pragma unroll
-    for (int i = 0; i < KT; ++i) u[i] = zs[__ldg(pi + i)];
-    // hidden units 8h .. 8h + 7: h_j = b1_j + sum_i W1[j][i] u_i, in input order
-    float2 hv[4];
-#pragma unroll
-    for (int m = 0; m < 4; ++m) hv[m] = make_float2(b1s[8 * h + 2 * m], b1s[8 * h + 2 * m + 1]);
-#pragma unroll
-    for (int i = 0; i < KT; ++i) {
-        const float2 uu = make_float2(u[i], u[i]);
-        const float4 wa = W1t[4 * i + 2 * h], wb = W1t[4 * i + 2 * h + 1];
-        hv[0] = __ffma2_rn(make_float2(wa.x, wa.y), uu, hv[0]);
-        hv[1] = __ffma2_rn(make_float2(wa.z, wa.w), uu, hv[1]);
-        hv[2] = __ffma2_rn(make_float2(wb.x, wb.y), uu, hv[2]);
-        hv[3] = __ffma2_rn(make_float2(wb.z, wb.w), uu, hv[3]);
-    }
-    float gp = 0.f;
-#pragma unroll
-    for (int m = 0; m < 4; ++m) {
-        gp = fmaf(w2s[8 * h + 2 * m], fmaxf(hv[m].x, 0.f), gp);
-        gp = fmaf(w2s[8 * h + 2 * m + 1], fmaxf(hv[m].y, 0.f), gp);
-    }
-    const float go = __shfl_xor_sync(0xffffffffu, gp, 1);
-    const float g = (h ? go + gp : gp + go) + __ldg(P.b2);
-    const float tau = P.tmin + (P.tmax - P.tmin) / (1.f + expf(-g));
-    // a_i = exp((L_i - L_0) / tau) / sum_j exp((L_j - L_0) / tau)
-    const float L0 = __ldg(pl);  // position 0 holds the largest logit
-    const float rt = 1.f / tau;
-    float ex[8], sp = 0.f;
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-        const int i = 8 * h + m;
-        ex[m] = i < k ? expf((__ldg(pl + i) - L0) * rt) : 0.f;
-        sp += ex[m];
-    }
-    const float so = __shfl_xor_sync(0xffffffffu, sp, 1);
-    const float S = h ? so + sp : sp + so;
-    const float inv = 1.f / S;
-    if (act) {
-        float4 *wt = reinterpret_cast<float4 *>(P.wblk + (size_t)n * (P.tb_bytes >> 2) + wofs(e) + 8 * h);
-        wt[0] = make_float4(ex[0] * inv, ex[1] * inv, ex[2] * inv, ex[3] * inv);
-        wt[1] = make_float4(ex[4] * inv, ex[5] * inv, ex[6] * inv, ex[7] * inv);
-        if (h == 0) P.tau[(size_t)n * P.R + e] = tau;
-    }
-    // the weights, z and tau are visible before the tag
-    __threadfence();
-    bar_sync(kBarGate, 128);
-    if (gt == 0) st_release(P.flag + n, tag);
-    return true;
-}
-
-// Gate role: the examples whose last tile is one of this CTA's items, in order.
-template <int KT>
-__device__ void role_gate(const StreamParams &P, unsigned char *sm, uint32_t tag) {
-    const int nj = items_of_cta(P);
-    for (int j = 0; j < nj; ++j) {
-        const Item I = item_of(P, j);
-        if (I.t != P.T - 1) continue;
-        if (!gate_example<KT>(P, sm, I.n, tag, I.it)) break;
+        // every thread's weights, z and tau are visible before the tag (the
+        // barrier orders them before thread 0's fence, which is cumulative)
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            st_release(P.flag + n, tag);
+        }
     }
 }
 
-// Table + store: for item j, the weights of its example (waiting, bounded,
-// for the tag its gate publishes) into table j mod kNT; then the staged y
-// tile of item j - 1 leaves by one bulk copy (its 16-byte aligned body) and
-// plain stores (the unaligned head and tail, under 16 bytes each), and the
-// staging buffer is handed back once the copy has read it. The table of
-// item j never waits for a store, so the two duties share the warp without
-// a cycle of waits.
-__device__ void role_table_store(const StreamParams &P, unsigned char *sm, uint32_t tag) {
+// Store: the staged y tile of item j (buffer j mod kNY) leaves by one bulk
+// copy (its 16-byte aligned body) and plain stores (the unaligned head and
+// tail, under 16 bytes each); the buffer goes back to the mix warps as soon
+// as the copy has read it.
+__device__ void role_store(const StreamParams &P, unsigned char *sm) {
     const int lane = threadIdx.x & 31;
     const uint32_t bar = smem_u32(sm + P.off_bar);
     const int Rp = P.R + 1;
-    const int n16 = (int)(P.tb_bytes >> 4);
     const int nj = items_of_cta(P);
-    for (int j = 0; j <= nj; ++j) {
-        if (j < nj) {
-            const Item I = item_of(P, j);
-            const int q = j % kNT;
-            bool ok = j < kNT || mbar_wait(bar + 8u * (kMbTFree + q), (uint32_t)((j / kNT) - 1) & 1u,
-                                           P.ctrl, I.it);
-            if (ok && lane == 0) {
-                ok = false;
-                for (uint32_t i = 0; i < kSpinLimit; ++i) {
-                    if (ld_acquire(P.flag + I.n) == tag) { ok = true; break; }
-                    if ((i & 15u) == 15u && ld_relaxed(P.ctrl + kCtrlError) != 0u) break;
-                    __nanosleep(i < 64 ? 20 : 200);
-                }
-                if (!ok && ld_relaxed(P.ctrl + kCtrlError) == 0u) report_timeout(P.ctrl, I.it);
-            }
-            if (!__shfl_sync(0xffffffffu, ok, 0)) break;
-            const uint4 *src =
-                reinterpret_cast<const uint4 *>(P.wblk + (size_t)I.n * (P.tb_bytes >> 2));
-            uint4 *dst = reinterpret_cast<uint4 *>(sm + P.off_tab + (size_t)q * P.tb_bytes);
-            for (int i = lane; i < n16; i += 32) dst[i] = __ldcg(src + i);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar + 8u * (kMbTReady + q));
+    for (int j = 0; j < nj; ++j) {
+        const Item I = item_of(P, j);
+        const int b = j % kNY;
+        if (!__all_sync(0xffffffffu, mbar_wait(bar + 8u * (kMbYDone + b),
+                                                (uint32_t)(j / kNY) & 1u, P.ctrl, I.it)))
+            break;  // warp-uniform exit
+        uint16_t *ydst = P.y + ((size_t)I.n * P.HW + (size_t)I.t * kTP) * Rp;
+        const uint32_t dmis = (uint32_t)(reinterpret_cast<uintptr_t>(ydst) & 15u);
+        const uint16_t *ys =
+            reinterpret_cast<const uint16_t *>(sm + P.off_ys + (size_t)b * P.ysb + dmis);
+        // byte offsets from ydst: [0, a0) head, [a0, a1) body, [a1, nbytes) tail
+        const uint32_t nbytes = (uint32_t)I.valid * (uint32_t)Rp * 2u;
+        const uint32_t hi = (dmis + nbytes) & ~15u;
+        const uint32_t a0 = min((16u - dmis) & 15u, nbytes);
+        const uint32_t a1 = max(a0, hi - min(dmis, hi));
+        if (lane == 0 && a1 > a0)
+            bulk_store(reinterpret_cast<unsigned char *>(ydst) + a0,
+                       smem_u32(reinterpret_cast<const unsigned char *>(ys) + a0), a1 - a0);
+        if (lane < 8) {
+            const uint32_t e = (uint32_t)lane;
+            if (2u * e < a0) ydst[e] = ys[e];
+            const uint32_t te = (a1 >> 1) + e;
+            if (2u * te < nbytes) ydst[te] = ys[te];
         }
-        if (j > 0) {
-            const int js = j - 1;
-            const Item I = item_of(P, js);
-            if (!__all_sync(0xffffffffu,
-                            mbar_wait(bar + 8u * kMbYDone, (uint32_t)js & 1u, P.ctrl, I.it)))
-                break;  // warp-uniform exit
-            uint16_t *ydst = P.y + ((size_t)I.n * P.HW + (size_t)I.t * kTP) * Rp;
-            const uint32_t dmis = (uint32_t)(reinterpret_cast<uintptr_t>(ydst) & 15u);
-            const uint16_t *ys = reinterpret_cast<const uint16_t *>(sm + P.off_ys + dmis);
-            // byte offsets from ydst: [0, a0) head, [a0, a1) body, [a1, nbytes) tail
-            const uint32_t nbytes = (uint32_t)I.valid * (uint32_t)Rp * 2u;
-            const uint32_t hi = (dmis + nbytes) & ~15u;
-            const uint32_t a0 = min((16u - dmis) & 15u, nbytes);
-            const uint32_t a1 = max(a0, hi - min(dmis, hi));
-            if (lane == 0 && a1 > a0)
-                bulk_store(reinterpret_cast<unsigned char *>(ydst) + a0,
-                           smem_u32(reinterpret_cast<const unsigned char *>(ys) + a0), a1 - a0);
-            if (lane < 8) {
-                const uint32_t e = (uint32_t)lane;
-                if (2u * e < a0) ydst[e] = ys[e];
-                const uint32_t te = (a1 >> 1) + e;
-                if (2u * te < nbytes) ydst[te] = ys[te];
-            }
-            if (lane == 0) bulk_wait_read<0>();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar + 8u * kMbYFree);
+        // the buffer goes back once the copy has read it
+        if (lane == 0) {
+            bulk_wait_read<0>();
+            mbar_arrive(bar + 8u * (kMbYFree + b));
         }
+        __syncwarp();
     }
     if (lane == 0) bulk_wait_all();
 }
@@ -678,15 +788,14 @@ __device__ void role_mix(const StreamParams &P, unsigned char *sm) {
     const int pair = (w & 3) + 16 * (w >> 2) + 4 * G4;
     const int e0 = 2 * pair, e1 = e0 + 1;
     const bool v0 = e0 < P.R, v1 = e1 < P.R;
-    constexpr int k = KT;
     const uint32_t bar = smem_u32(sm + P.off_bar);
-    const uint32_t xs0 = smem_u32(sm + P.off_x);
+    const uint32_t xs0 = smem_u32(sm + P.off_mix);
     const uint32_t sb = (uint32_t)P.C * kTP * 2u;
     uint32_t off0[KT], off1[KT];
 #pragma unroll
     for (int i = 0; i < KT; ++i) {
-        const int c0 = v0 ? __ldg(P.pidx + e0 * k + i) : 0;
-        const int c1 = v1 ? __ldg(P.pidx + e1 * k + i) : 0;
+        const int c0 = v0 ? __ldg(P.pidx + e0 * KT + i) : 0;
+        const int c1 = v1 ? __ldg(P.pidx + e1 * KT + i) : 0;
         off0[i] = (uint32_t)c0 * 128u + ((uint32_t)(jc ^ ((c0 & 1) << 2)) << 4);
         off1[i] = (uint32_t)c1 * 128u + ((uint32_t)(jc ^ ((c1 & 1) << 2)) << 4);
     }
@@ -694,8 +803,8 @@ __device__ void role_mix(const StreamParams &P, unsigned char *sm) {
     const int nj = items_of_cta(P);
     for (int j = 0; j < nj; ++j) {
         const Item I = item_of(P, j);
-        const int s = j % P.D, q = j % kNT;
-        bool ok = mbar_wait(bar + 8u * (kMbStaged + s), (uint32_t)(j / P.D) & 1u, P.ctrl, I.it);
+        const int s = j % P.DM, q = j % kNT;
+        bool ok = mbar_wait(bar + 8u * (kMbStaged + s), (uint32_t)(j / P.DM) & 1u, P.ctrl, I.it);
         ok = ok && mbar_wait(bar + 8u * (kMbTReady + q), (uint32_t)(j / kNT) & 1u, P.ctrl, I.it);
         if (!__all_sync(0xffffffffu, ok)) break;  // warp-uniform exit
         // the pair's weights of this example
@@ -737,13 +846,22 @@ __device__ void role_mix(const StreamParams &P, unsigned char *sm) {
             b[2] = __ffma2_rn(c1, unpack2(x1.z), b[2]);
             b[3] = __ffma2_rn(c1, unpack2(x1.w), b[3]);
         }
-        // y tile: [positions][R + 1] bf16 in the staging buffer, placed so that
-        // it has the alignment mod 16 of its destination in y
+        // the residual partials of the channel groups, in group order
+        float rv = 0.f;
+        if (tid < kTP)
+            for (int g = 0; g < P.nreg; ++g) rv += res_part(P, sm, s, g)[tid];
+        // the slot is read: it goes back to the mix producer
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar + 8u * (kMbEmpty + s));
+        // y tile: [positions][R + 1] bf16 in staging buffer j mod kNY, placed so
+        // that it has the alignment mod 16 of its destination in y
+        const int yb = j % kNY;
         const size_t row0 = (size_t)I.n * P.HW + (size_t)I.t * kTP;
         const uint32_t dmis = (uint32_t)(reinterpret_cast<uintptr_t>(P.y + row0 * Rp) & 15u);
-        uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys + dmis);
-        // the store of item j - 1 has read the staging buffer
-        ok = j < 1 || mbar_wait(bar + 8u * kMbYFree, (uint32_t)(j - 1) & 1u, P.ctrl, I.it);
+        uint16_t *ys = reinterpret_cast<uint16_t *>(sm + P.off_ys + (size_t)yb * P.ysb + dmis);
+        // the store of item j - kNY has read the staging buffer
+        ok = j < kNY || mbar_wait(bar + 8u * (kMbYFree + yb), (uint32_t)((j / kNY) - 1) & 1u,
+                                  P.ctrl, I.it);
         if (!__all_sync(0xffffffffu, ok)) break;
 #pragma unroll
         for (int m = 0; m < 4; ++m) {
@@ -757,31 +875,26 @@ __device__ void role_mix(const StreamParams &P, unsigned char *sm) {
                 ys[(p + 1) * Rp + e1] = f32_to_bf16(b[m].y);
             }
         }
-        if (tid < kTP) {  // mix warps 0, 1: the residual column, once it is summed
-            ok = mbar_wait(bar + 8u * (kMbResDone + s), (uint32_t)(j / P.D) & 1u, P.ctrl, I.it);
-            if (!__all_sync(0xffffffffu, ok)) break;
-            ys[tid * Rp + P.R] = f32_to_bf16(res_of(P, sm, s)[tid]);
-        }
+        if (tid < kTP) ys[tid * Rp + P.R] = f32_to_bf16(rv * P.inv_nU);
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) {
-            mbar_arrive(bar + 8u * (kMbEmpty + s));
-            mbar_arrive(bar + 8u * kMbYDone);
-        }
+        if (lane == 0) mbar_arrive(bar + 8u * (kMbYDone + yb));
     }
 }
 
+// Stream CTA: barriers, U, then the roles.
 template <int KT>
-__global__ void __launch_bounds__(kThreads_, 1)
-    moce_stream_kernel(const __grid_constant__ CUtensorMap tmx, const StreamParams P) {
-    extern __shared__ unsigned char smraw[];
-    unsigned char *sm = smraw + ((1024u - (smem_u32(smraw) & 1023u)) & 1023u);
+__device__ void stream_cta(const StreamParams &P, const CUtensorMap *tm, unsigned char *sm,
+                           uint32_t tag) {
     const int tid = threadIdx.x, warp = tid >> 5;
-    const uint32_t tag = ld_relaxed(P.ctrl + kCtrlEpoch) + 1u;
     if (tid == 0) {
         const uint32_t bar = smem_u32(sm + P.off_bar);
-        for (int d = 0; d < P.D; ++d) {
-            mbar_init(bar + 8u * (kMbRaw + d), 1);
+        for (int d = 0; d < kDP; ++d) {
+            mbar_init(bar + 8u * (kMbPRaw + d), 1);
+            mbar_init(bar + 8u * (kMbPFree + d), 1);
+        }
+        for (int d = 0; d < P.DM; ++d) {
+            mbar_init(bar + 8u * (kMbMRaw + d), 1);
             mbar_init(bar + 8u * (kMbStaged + d), 4);
             mbar_init(bar + 8u * (kMbEmpty + d), kMixT / 32);
         }
@@ -789,52 +902,81 @@ __global__ void __launch_bounds__(kThreads_, 1)
             mbar_init(bar + 8u * (kMbTReady + q), 1);
             mbar_init(bar + 8u * (kMbTFree + q), kMixT / 32);
         }
-        mbar_init(bar + 8u * kMbYDone, kMixT / 32);
-        mbar_init(bar + 8u * kMbYFree, 1);
-        for (int q = 0; q < 2; ++q) {
-            mbar_init(bar + 8u * (kMbPooled + q), 4);
-            mbar_init(bar + 8u * (kMbPFree + q), 1);
+        for (int b = 0; b < kNY; ++b) {
+            mbar_init(bar + 8u * (kMbYDone + b), kMixT / 32);
+            mbar_init(bar + 8u * (kMbYFree + b), 1);
         }
-        for (int d = 0; d < P.D; ++d) mbar_init(bar + 8u * (kMbResDone + d), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(bar + 8u * (kMbPooled + b), 1);
+            mbar_init(bar + 8u * (kMbPsFree + b), 1);
+        }
+        st_ctr(ctr_addr(P, sm, 0), 0u);
+        st_ctr(ctr_addr(P, sm, 1), 0u);
         fence_mbar_init();
     }
-    // resident tables: U and the gate parameters (W1 transposed, zero-padded
-    // to 16 x 16; b1 and w2 zero-padded to 16)
-    {
-        uint16_t *Us = reinterpret_cast<uint16_t *>(sm + P.off_U);
-        for (int i = tid; i < P.nU; i += kThreads_) Us[i] = (uint16_t)__ldg(P.resid + i);
-        float *W1t = reinterpret_cast<float *>(sm + P.off_w1t);
-        for (int q = tid; q < kKMax * kKMax; q += kThreads_) {
-            const int i = q / kKMax, jh = q % kKMax;
-            W1t[q] = (i < P.k && jh < P.k) ? __ldg(P.W1 + jh * P.k + i) : 0.f;
-        }
-        for (int i = tid; i < kKMax; i += kThreads_) {
-            reinterpret_cast<float *>(sm + P.off_b1)[i] = i < P.k ? __ldg(P.b1 + i) : 0.f;
-            reinterpret_cast<float *>(sm + P.off_w2)[i] = i < P.k ? __ldg(P.w2 + i) : 0.f;
-        }
-        // the accumulator bank of the previous (and the next) forward
-        unsigned long long *other = P.zacc + (size_t)(tag & 1u) * P.N * P.C;
-        const size_t nw = (size_t)P.N * P.C;
-        for (size_t i = (size_t)blockIdx.x * kThreads_ + tid; i < nw; i += (size_t)gridDim.x * kThreads_)
-            other[i] = 0ull;
-    }
+    uint16_t *Us = reinterpret_cast<uint16_t *>(sm + P.off_U);
+    for (int i = tid; i < P.nU; i += kThreads_) Us[i] = (uint16_t)__ldg(P.resid + i);
     __syncthreads();
     if (warp < 4) {
+        set_role_regs<kRegPool, kRegLaunch>();
+        role_pool(P, sm);
+    } else if (warp < 8) {
         set_role_regs<kRegTr, kRegLaunch>();
         role_transpose(P, sm);
-    } else if (warp < 8) {
-        set_role_regs<kRegGate, kRegLaunch>();
-        role_gate<KT>(P, sm, tag);
     } else if (warp < 16) {
         set_role_regs<kRegMix, kRegLaunch>();
         role_mix<KT>(P, sm);
     } else {
         set_role_regs<kRegMisc, kRegLaunch>();
-        if (warp == kProdW) role_producer(P, &tmx, sm);
-        else if (warp == kStoreW) role_table_store(P, sm, tag);
-        else if (warp == kPubW) role_publish(P, sm);
-        else if (warp == kResW) role_residual(P, sm);
+        if (warp == kPoolProdW) role_pool_producer(P, tm, sm);
+        else if (warp == kMixProdW) role_mix_producer(P, tm, sm, tag);
+        else if (warp == kStoreW) role_store(P, sm);
+        else role_publish(P, sm);
     }
+}
+
+// Gate CTA: the resident gate parameters, then its examples.
+template <int KT>
+__device__ void gate_cta_main(const StreamParams &P, unsigned char *sm, uint32_t tag) {
+    const int tid = threadIdx.x;
+    float *W1t = reinterpret_cast<float *>(sm + P.g_w1t);
+    for (int q = tid; q < kKMax * kKMax; q += kThreads_) {
+        const int i = q / kKMax, jh = q % kKMax;
+        W1t[q] = (i < KT && jh < KT) ? __ldg(P.W1 + jh * KT + i) : 0.f;
+    }
+    for (int i = tid; i < kKMax; i += kThreads_) {
+        reinterpret_cast<float *>(sm + P.g_b1)[i] = i < KT ? __ldg(P.b1 + i) : 0.f;
+        reinterpret_cast<float *>(sm + P.g_w2)[i] = i < KT ? __ldg(P.w2 + i) : 0.f;
+    }
+    uint16_t *gidx = reinterpret_cast<uint16_t *>(sm + P.g_idx);
+    float *gdl = reinterpret_cast<float *>(sm + P.g_dl);
+    for (int q = tid; q < P.R * kKMax; q += kThreads_) {
+        const int e = q / kKMax, i = q % kKMax;
+        gidx[q] = i < KT ? (uint16_t)__ldg(P.pidx + e * KT + i) : 0;
+        gdl[q] = i < KT ? __ldg(P.plog + e * KT + i) - __ldg(P.plog + e * KT) : 0.f;
+    }
+    __syncthreads();
+    gate_cta<KT>(P, sm, tag);
+}
+
+// CTAs 0 .. Gs - 1 stream the items; CTAs Gs .. Gs + Gg - 1 run the gates.
+template <int KT>
+__global__ void __launch_bounds__(kThreads_, 1)
+    moce_stream_kernel(const __grid_constant__ CUtensorMap tmx, const StreamParams P) {
+    extern __shared__ unsigned char smraw[];
+    unsigned char *sm = smraw + ((1024u - (smem_u32(smraw) & 1023u)) & 1023u);
+    const int tid = threadIdx.x;
+    const uint32_t tag = ld_relaxed(P.ctrl + kCtrlEpoch) + 1u;
+    {
+        // the accumulator bank of the previous (and the next) forward
+        unsigned long long *other = P.zacc + (size_t)(tag & 1u) * P.N * P.C;
+        const size_t nw = (size_t)P.N * P.C;
+        for (size_t i = (size_t)blockIdx.x * kThreads_ + tid; i < nw;
+             i += (size_t)gridDim.x * kThreads_)
+            other[i] = 0ull;
+    }
+    if ((int)blockIdx.x < P.Gs) stream_cta<KT>(P, &tmx, sm, tag);
+    else gate_cta_main<KT>(P, sm, tag);
     __syncthreads();
     if (tid == 0) {
         // the last CTA to finish advances the epoch for the next forward
@@ -876,6 +1018,18 @@ struct StreamPlan {
     size_t smem = 0;
 };
 
+// Items the pool stream may run ahead of the mix stream's loads: enough to
+// cover the latency from a tile's pooling to its example's weights, few
+// enough that the lines it has read stay in L2 until the mix stream reads
+// them (Gs (lead + pool slots) tiles, about 66 MB at 148 stream CTAs and
+// C_in 256; on the 256-channel, 64-example layer leads of 10 to 22 measure
+// alike, 6 is 12 % slower).
+constexpr int kLead = MOCE_STREAM_LEAD;
+// Items the pool producer prefetches into L2 ahead of its loads.
+constexpr int kPrefetch = MOCE_STREAM_PF;
+// SMs that run gates only.
+constexpr int kGateCtas = 4;
+
 bool plan_stream(int N, int HW, int C, int R, int k, int sms, StreamPlan *out) {
     if (C < 64 || C > 256 || C % 64 != 0 || R < 1 || R > kRMax || k < 1 || k > kKMax) return false;
     if (N < 1 || HW < 1 || sms < 1) return false;
@@ -892,7 +1046,11 @@ bool plan_stream(int N, int HW, int C, int R, int k, int sms, StreamPlan *out) {
     const long long items = (long long)N * p.T;
     if (items > 0x7fffffffll) return false;
     p.items = (uint32_t)items;
-    p.G = (int)std::min<long long>(sms, items);
+    // a few whole SMs run the gates: on a stream SM they would share the issue
+    // slots and shared memory with the mixing and come late
+    p.Gg = std::min(kGateCtas, N);
+    if (sms <= p.Gg) return false;
+    p.Gs = (int)std::min<long long>(sms - p.Gg, items);
     p.nreg = C / 64;
     p.tb_bytes = table_bytes(R);
     p.ysb = (uint32_t)align_up((size_t)kTP * (R + 1) * 2, 16) + 16u;
@@ -904,31 +1062,47 @@ bool plan_stream(int N, int HW, int C, int R, int k, int sms, StreamPlan *out) {
         return (uint32_t)o;
     };
     p.off_tab = take((size_t)kNT * p.tb_bytes, 16);
-    p.off_ys = take((size_t)p.ysb, 16);
-    p.off_res = take((size_t)kMaxD * kTP * 4, 16);
+    p.off_ys = take((size_t)kNY * p.ysb, 16);
     p.off_U = take((size_t)C * 2, 16);
-    p.off_zs = take((size_t)C * 4, 16);
-    p.off_w1t = take((size_t)kKMax * kKMax * 4, 16);
-    p.off_b1 = take((size_t)kKMax * 4, 16);
-    p.off_w2 = take((size_t)kKMax * 4, 16);
+    p.off_Ur = take((size_t)4 * C * 2, 16);
     p.off_psum = take((size_t)2 * C * 4, 16);
     p.off_pword = take((size_t)2 * C * 8, 16);
+    p.off_ctr = take(16, 16);
     p.off_bar = take((size_t)kMbCount * 8, 8);
-    const size_t fixed = align_up(off, 1024);
-    const size_t sb = (size_t)kTP * C * 2;
+    // the residual partials: 4 groups x 64 positions of fp32 per mix slot
+    const size_t sb = (size_t)kTP * C * 2, resb = (size_t)4 * kTP * 4;
     const size_t budget = 227 * 1024 - 1024;  // 1 KB for aligning the dynamic base
-    if (fixed + 3 * sb > budget) return false;
-    p.D = (int)std::min<size_t>(kMaxD, (budget - fixed) / sb);
-    // an example's tiles span ceil(T / G) + 1 rounds at most: with D slots a
-    // CTA can hold what the gates of its oldest item still wait for
-    if ((p.G - 1 + p.T - 1) / p.G > p.D - 1) return false;
+    p.DM = 0;
+    for (int dm = kMaxDM; dm >= 2 && p.DM == 0; --dm)
+        if (align_up(align_up(off, 16) + dm * resb, 1024) + (kDP + dm) * sb <= budget) p.DM = dm;
+    if (p.DM == 0) return false;
+    p.off_res = take((size_t)p.DM * resb, 16);
+    const size_t fixed_end = off;
+    p.lead = kLead;
+    p.PF = kPrefetch;
+    // Progress: the pool stream's item j waits for the mix producer to load
+    // item j - lead, which it does after the weights of item j - lead - 1's
+    // example are published. That example must be an earlier one than every
+    // example item j belongs to, so (lead + 1) Gs must exceed the tiles of one
+    // example (with one round to spare).
+    if ((long long)p.lead * p.Gs < (long long)p.T) return false;
     // slots first (1024-aligned for the 128-byte swizzle), then the rest
-    const uint32_t shift = (uint32_t)(p.D * sb);
-    p.off_x = 0;
-    for (uint32_t *o : {&p.off_tab, &p.off_ys, &p.off_res, &p.off_U, &p.off_zs, &p.off_w1t,
-                        &p.off_b1, &p.off_w2, &p.off_psum, &p.off_pword, &p.off_bar})
+    p.off_pool = 0;
+    p.off_mix = (uint32_t)(kDP * sb);
+    const uint32_t shift = (uint32_t)((kDP + p.DM) * sb);
+    for (uint32_t *o : {&p.off_tab, &p.off_ys, &p.off_U, &p.off_Ur, &p.off_psum, &p.off_pword,
+                        &p.off_ctr, &p.off_bar, &p.off_res})
         *o += shift;
-    p.smem_bytes = (uint32_t)(shift + off + 1024);
+    // the gate CTAs' resident tables, from the start of shared memory
+    off = 0;
+    p.g_zs = take((size_t)C * 4, 16);
+    p.g_w1t = take((size_t)kKMax * kKMax * 4, 16);
+    p.g_b1 = take((size_t)kKMax * 4, 16);
+    p.g_w2 = take((size_t)kKMax * 4, 16);
+    p.g_idx = take((size_t)R * kKMax * 2, 16);
+    p.g_dl = take((size_t)R * kKMax * 4, 16);
+    if (off > shift) return false;  // never: the slots alone exceed it
+    p.smem_bytes = (uint32_t)(shift + fixed_end + 1024);
     out->smem = p.smem_bytes;
     return true;
 }
@@ -949,12 +1123,17 @@ cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
     if (!plan_stream(N, HW, C, R, k, sm_count(), &plan)) return cudaErrorNotSupported;
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
+    // x viewed as [channel group][example][position][64 channels]: one box
+    // of {64, 64, 1, C / 64} is a whole tile, landing as C / 64 regions of
+    // [64 positions][128 bytes] (128-byte swizzle) in one copy (copies of
+    // 32 KB keep HBM busy where 8 KB ones, a box per channel group, do not);
+    // positions past the example's HW are outside the view and read as zeros.
     CUtensorMap tm;
-    const cuuint64_t dims[2] = {(cuuint64_t)C, (cuuint64_t)N * (cuuint64_t)HW};
-    const cuuint64_t strides[1] = {(cuuint64_t)C * 2};
-    const cuuint32_t box[2] = {64, kTP};
-    const cuuint32_t es[2] = {1, 1};
-    if (enc(&tm, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t *>(x), dims, strides, box,
+    const cuuint64_t dims[4] = {64, (cuuint64_t)HW, (cuuint64_t)N, (cuuint64_t)(C / 64)};
+    const cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)HW * C * 2, 128};
+    const cuuint32_t box[4] = {64, kTP, 1, (cuuint32_t)(C / 64)};
+    const cuuint32_t es[4] = {1, 1, 1, 1};
+    if (enc(&tm, CU_TENSOR_MAP_DATA_TYPE_UINT16, 4, const_cast<uint16_t *>(x), dims, strides, box,
             es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorInvalidValue;
@@ -1002,7 +1181,7 @@ cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
         }
     }
     void *args[] = {&tm, &P};
-    return cudaLaunchCooperativeKernel((const void *)kern, dim3(P.G), dim3(kThreads_), args,
+    return cudaLaunchCooperativeKernel((const void *)kern, dim3(P.Gs + P.Gg), dim3(kThreads_), args,
                                        plan.smem, s);
 }
 
