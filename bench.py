@@ -51,7 +51,7 @@ def parse_args():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto",
-                    help="kernel path of the forward (auto, two_pass, pipe, ring, fused, steps)")
+                    help="kernel path of the forward (auto, stream, steps)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline leg")
     return ap.parse_args()

@@ -20,7 +20,8 @@
  * Conventions shared by every entry point:
  *   - All tensor pointers are DEVICE pointers unless the name ends in _host.
  *     The caller owns every buffer; the library never allocates memory and
- *     keeps no global state.
+ *     keeps no global state, with one exception: moce_forward_noalloc uses a
+ *     fixed scratch array in the library's device image (see there).
  *   - Calls are asynchronous on `stream` unless stated otherwise. A NULL
  *     stream is the legacy default stream.
  *   - Arguments are validated on the host before any launch; an invalid
@@ -58,38 +59,25 @@ typedef enum moce_dtype { MOCE_F32 = 0, MOCE_BF16 = 1 } moce_dtype_t;
 typedef enum moce_layout { MOCE_NHWC = 0, MOCE_NCHW = 1 } moce_layout_t;
 
 /*
- * Kernel path of one layer forward (moce_forward_path). Every path computes
- * the same layer (Sec. 3.2-3.4) and gives the same results within bf16
- * output rounding; they differ in how x travels through the GPU.
- *   MOCE_PATH_AUTO      the fastest path that supports the arguments
- *                       (TWO_PASS, else PIPE, else FUSED, else STEPS)
- *   MOCE_PATH_PIPE      one warp-specialised persistent kernel (NHWC bf16,
- *                       8 <= C_in <= 256, C_in % 8 == 0, k <= 16)
- *   MOCE_PATH_TWO_PASS  a pooling+gate kernel, then a mixing kernel that
- *                       stages x through a shared-memory ring (NHWC bf16,
- *                       as PIPE and C_out <= 64)
- *   MOCE_PATH_FUSED     the two-group persistent kernel (NHWC bf16,
- *                       C_in % 8 == 0, k <= 16, shared memory permitting)
- *   MOCE_PATH_STEPS     one kernel per step: pool, gate, mix (any layout
- *                       and dtype)
- *   MOCE_PATH_RING      one cooperative kernel in which every CTA pools its
- *                       tiles a few rounds before it mixes them and the CTA
- *                       that pools an example's last tile runs the gate
- *                       (the shapes of TWO_PASS; correct, but slower than
- *                       TWO_PASS on the measured workloads)
- *   MOCE_PATH_STREAM    one cooperative kernel that reads x from HBM once:
- *                       each tile stays in shared memory from its pooling
- *                       until its example's gate has run (NHWC bf16,
- *                       64 <= C_in <= 256, C_in % 64 == 0, C_out <= 64,
- *                       k <= 16, x 16-byte aligned)
+ * Kernel path of one layer forward (moce_forward_path). Both paths compute
+ * the same layer (Sec. 3.2-3.4) and give the same results within bf16 output
+ * rounding; they differ in how x travels through the GPU.
+ *   MOCE_PATH_AUTO      STREAM when it supports the arguments, else STEPS
+ *   MOCE_PATH_STEPS     one kernel per step: pool, gate, mix (any layout and
+ *                       dtype); x is read twice
+ *   MOCE_PATH_STREAM    one cooperative kernel that reads x from HBM once: a
+ *                       pool stream reads each tile a few items ahead of a
+ *                       mix stream, which reads it again from L2 once its
+ *                       example's gate (run by a few dedicated CTAs) has
+ *                       published the weights (NHWC bf16, 64 <= C_in <= 256,
+ *                       C_in % 64 == 0, C_out <= 64, k <= 16, x 16-byte
+ *                       aligned)
+ * The values 1, 2, 3 and 5 belonged to kernels this library no longer has;
+ * asking for them returns MOCE_ERR_INVALID_VALUE.
  */
 typedef enum moce_path {
     MOCE_PATH_AUTO = 0,
-    MOCE_PATH_PIPE = 1,
-    MOCE_PATH_TWO_PASS = 2,
-    MOCE_PATH_FUSED = 3,
     MOCE_PATH_STEPS = 4,
-    MOCE_PATH_RING = 5,
     MOCE_PATH_STREAM = 6
 } moce_path_t;
 
@@ -193,12 +181,11 @@ moce_status_t moce_gate(const float *z, int N, int C_in, int C_out, int k,
  *   ws, ws_bytes: >= moce_workspace_bytes(N, H, W, C_in, C_out, k), 256-byte
  *   aligned, zero-filled before its first use (moce_workspace_init); one
  *   workspace serves one stream at a time.
- * NHWC bf16 with C_in % 8 == 0 and 16-byte aligned x runs the two-pass
- * path where it fits (C_in <= 256, C_out <= 64, k <= 16), else a persistent
- * kernel; other layouts/dtypes run a sequence of kernels (the choice is
- * moce_forward_path's MOCE_PATH_AUTO).
- * Asynchronous; device-side failures of the fused kernels (a bounded wait
- * that ran out) are reported by moce_check_device_error.
+ * NHWC bf16 with 16-byte aligned x runs the stream kernel where it fits
+ * (64 <= C_in <= 256, C_in % 64 == 0, C_out <= 64, k <= 16), else one kernel
+ * per step (the choice is moce_forward_path's MOCE_PATH_AUTO).
+ * Asynchronous; device-side failures (a bounded wait that ran out) are
+ * reported by moce_check_device_error.
  */
 moce_status_t moce_forward(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                            moce_dtype_t dtype, moce_layout_t layout, const int32_t *packed_idx,
@@ -239,6 +226,8 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
  *   - Every call shares the one array per device: each call clears the part
  *     it uses on `stream`, then runs the forward. Calls whose work overlaps on
  *     the GPU (other streams, other host threads) race on the array.
+ *   - Device-side failures (a bounded wait that ran out) are reported by
+ *     moce_noalloc_check_device_error, not by the return value.
  */
 moce_status_t moce_forward_noalloc(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                    moce_dtype_t dtype, moce_layout_t layout,
@@ -246,6 +235,15 @@ moce_status_t moce_forward_noalloc(const void *x, int N, int H, int W, int C_in,
                                    const int32_t *resid_idx, int n_resid, const float *W1,
                                    const float *b1, const float *w2, const float *b2,
                                    float tau_min, float tau_max, void *y, moce_stream_t stream);
+
+/*
+ * SYNCHRONOUS: waits for `stream`, then reads the device error word that the
+ * last moce_forward_noalloc on the current device left in the scratch array.
+ * MOCE_OK, MOCE_ERR_TIMEOUT (a bounded wait of that forward gave up; its y is
+ * invalid) or MOCE_ERR_CUDA. Each moce_forward_noalloc clears the word, so
+ * check before the next call on the device.
+ */
+moce_status_t moce_noalloc_check_device_error(moce_stream_t stream);
 
 /*
  * Number of kernel launches moce_forward makes for these arguments (the
@@ -257,19 +255,16 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
 
 /*
  * Name of the kernel path moce_forward takes for these arguments:
- * "moce_poolgate_kernel+moce_ring_kernel" (the two-pass path),
- * "moce_pipe_kernel" (the warp-specialised pipeline), "moce_fused_kernel"
- * (the two-group persistent kernel) or "pool+gate+mix" (one kernel per
- * step). NULL for arguments moce_forward would reject. Enqueues nothing; the
- * string is static.
+ * "moce_stream_kernel" (one cooperative kernel) or "pool+gate+mix" (one
+ * kernel per step). NULL for arguments moce_forward would reject. Enqueues
+ * nothing; the string is static.
  */
 const char *moce_forward_kernel(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                 moce_dtype_t dtype, moce_layout_t layout);
 
 /*
  * moce_forward_launches and moce_forward_kernel for moce_forward_path with
- * `path`: 0 / NULL where that path cannot run the arguments. The two-pass
- * path is named "moce_poolgate_kernel+moce_ring_kernel" (2 launches).
+ * `path`: 0 / NULL where that path cannot run the arguments.
  */
 int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                moce_dtype_t dtype, moce_layout_t layout, moce_path_t path);

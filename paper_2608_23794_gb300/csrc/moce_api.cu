@@ -135,26 +135,18 @@ static moce_path_t pick_path(const void *x, int N, int HW, int C_in, int C_out, 
                              moce_dtype_t dtype, moce_layout_t layout, moce_path_t want) {
     const bool vec = dtype == MOCE_BF16 && layout == MOCE_NHWC && C_in % 8 == 0 &&
                      (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
-    const bool pipe = vec && pipe_supported(N, HW, C_in, C_out, k);
-    const bool two = vec && ring_supported(N, HW, C_in, C_out, k, false);
-    const bool ring = vec && ring_supported(N, HW, C_in, C_out, k, true);
-    const bool fused = vec && fused_supported(N, HW, C_in, C_out, k);
     const bool stream = vec && stream_supported(N, HW, C_in, C_out, k);
     switch (want) {
-        case MOCE_PATH_AUTO:  // the fastest measured first
-            return stream ? MOCE_PATH_STREAM
-                   : two  ? MOCE_PATH_TWO_PASS
-                   : pipe ? MOCE_PATH_PIPE
-                   : fused ? MOCE_PATH_FUSED
-                           : MOCE_PATH_STEPS;
+        case MOCE_PATH_AUTO: return stream ? MOCE_PATH_STREAM : MOCE_PATH_STEPS;
         case MOCE_PATH_STREAM: return stream ? want : MOCE_PATH_AUTO;
-        case MOCE_PATH_PIPE: return pipe ? want : MOCE_PATH_AUTO;
-        case MOCE_PATH_TWO_PASS: return two ? want : MOCE_PATH_AUTO;
-        case MOCE_PATH_FUSED: return fused ? want : MOCE_PATH_AUTO;
         case MOCE_PATH_STEPS: return want;
-        case MOCE_PATH_RING: return ring ? want : MOCE_PATH_AUTO;
+        default: break;
     }
     return MOCE_PATH_AUTO;
+}
+
+static bool path_ok(moce_path_t p) {
+    return p == MOCE_PATH_AUTO || p == MOCE_PATH_STEPS || p == MOCE_PATH_STREAM;
 }
 
 moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, int C_out, int k,
@@ -165,7 +157,7 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
                                 float tau_max, void *y, void *ws, size_t ws_bytes,
                                 moce_path_t path, moce_stream_t stream) {
     if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
-        !tau_ok(tau_min, tau_max) || path < MOCE_PATH_AUTO || path > MOCE_PATH_STREAM)
+        !tau_ok(tau_min, tau_max) || !path_ok(path))
         return MOCE_ERR_INVALID_VALUE;
     if (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
     const int HW = H * W;
@@ -182,26 +174,10 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
     unsigned char *wsb = static_cast<unsigned char *>(ws);
     const uint16_t *xv = static_cast<const uint16_t *>(x);
     uint16_t *yv = static_cast<uint16_t *>(y);
-    switch (run) {
-        case MOCE_PATH_PIPE:
-            return cuda_status(launch_pipe(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
-                                           resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
-                                           yv, L, wsb, s));
-        case MOCE_PATH_TWO_PASS:
-        case MOCE_PATH_RING:
-            return cuda_status(launch_ring(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
-                                           resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
-                                           yv, L, wsb, run == MOCE_PATH_RING, s));
-        case MOCE_PATH_FUSED:
-            return cuda_status(launch_fused(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
-                                            resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
-                                            yv, L, wsb, s));
-        case MOCE_PATH_STREAM:
-            return cuda_status(launch_stream(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
-                                             resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max,
-                                             yv, L, wsb, s));
-        default: break;
-    }
+    if (run == MOCE_PATH_STREAM)
+        return cuda_status(launch_stream(xv, N, HW, C_in, C_out, k, packed_idx, packed_logits,
+                                         resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max, yv,
+                                         L, wsb, s));
     float *z = reinterpret_cast<float *>(wsb + L.z);
     float *tau = reinterpret_cast<float *>(wsb + L.tau);
     float *a = reinterpret_cast<float *>(wsb + L.a);
@@ -211,7 +187,7 @@ moce_status_t moce_forward_path(const void *x, int N, int H, int W, int C_in, in
                           tau_max, tau, a, s);
     if (err == cudaSuccess)
         err = launch_mix(x, N, HW, C_in, C_out, k, dtype, layout, packed_idx, a, resid_idx,
-                         n_resid, y, s);
+                         n_resid, y, reinterpret_cast<uint32_t *>(wsb + L.ctrl), s);
     return cuda_status(err);
 }
 
@@ -234,16 +210,12 @@ int moce_forward_launches(const void *x, int N, int H, int W, int C_in, int C_ou
 int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int C_out, int k,
                                moce_dtype_t dtype, moce_layout_t layout, moce_path_t path) {
     if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
-        path < MOCE_PATH_AUTO || path > MOCE_PATH_STREAM)
+        !path_ok(path))
         return 0;
     if (N == 0 || H * W == 0) return 0;
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
     switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
-        case MOCE_PATH_PIPE:
-        case MOCE_PATH_FUSED:
-        case MOCE_PATH_STREAM:
-        case MOCE_PATH_RING: return 1;
-        case MOCE_PATH_TWO_PASS: return 2;  // pool+gate, then mix
+        case MOCE_PATH_STREAM: return 1;
         case MOCE_PATH_STEPS: return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
         default: return 0;
     }
@@ -260,11 +232,7 @@ const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_i
     if (moce_forward_path_launches(x, N, H, W, C_in, C_out, k, dtype, layout, path) == 0)
         return nullptr;
     switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
-        case MOCE_PATH_PIPE: return "moce_pipe_kernel";
-        case MOCE_PATH_TWO_PASS: return "moce_poolgate_kernel+moce_ring_kernel";
-        case MOCE_PATH_FUSED: return "moce_fused_kernel";
         case MOCE_PATH_STEPS: return "pool+gate+mix";
-        case MOCE_PATH_RING: return "moce_ring_kernel";
         case MOCE_PATH_STREAM: return "moce_stream_kernel";
         default: return nullptr;
     }

@@ -1,6 +1,5 @@
 // Temperature gate, Eq. (tau), and mixing weights, Eq. (weights), for one
-// block of experts of one example. Shared by the standalone gate kernel and
-// the fused forward kernel.
+// block of experts of one example, for the standalone gate kernel (any k).
 //
 // For each (example n, routed expert e) the gate input is u = z[n, S_e] in
 // deployment order (position i = the expert's i-th most preferred channel,
@@ -29,8 +28,7 @@ __host__ __device__ inline size_t gate_smem(int k) {
 }
 
 // One block of GE experts of example n: 256 threads = GE experts x 8 threads
-// (4 hidden units each). gsm: gate_smem(k) bytes of shared memory. z is read
-// through L2 (__ldcg) because the fused kernel produces it in the same launch.
+// (4 hidden units each). gsm: gate_smem(k) bytes of shared memory.
 __device__ __forceinline__ void gate_block(float *gsm, int n, int e0, const float *__restrict__ z,
                                            int C, int R, int k, const int32_t *__restrict__ pidx,
                                            const float *__restrict__ plog,

@@ -10,15 +10,15 @@
 
 namespace moce {
 
-constexpr int kThreads = 256;  // threads of the standalone kernels and of the fused kernel's mix group
+constexpr int kThreads = 256;  // threads of the step kernels
 
 __host__ __device__ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 // ---------------------------------------------------------------- workspace
 // Control words at the start of a forward workspace.
 enum CtrlWord : int {
-    kCtrlExitCounter = 0,  // CTAs that finished the fused kernel
-    kCtrlEpoch = 1,        // number of completed fused forwards (data tags are epoch + 1)
+    kCtrlExitCounter = 0,  // CTAs that finished the stream kernel
+    kCtrlEpoch = 1,        // number of completed stream forwards (data tags are epoch + 1)
     kCtrlError = 2,        // 0, or kErrTimeout
     kCtrlErrorItem = 3,    // 1 + the work item whose wait gave up
     kCtrlDropItem = 4,     // fault injection for tests: 1 + a work item that must not publish
@@ -26,8 +26,6 @@ enum CtrlWord : int {
 };
 constexpr uint32_t kErrTimeout = 1u;
 
-// Experts per gate work item of the fused kernel.
-constexpr int kGateExperts = 64;
 
 // Pixels per pooling tile: about 32 KB of bf16 input per tile.
 inline int pool_tile_px(int C) {
@@ -37,36 +35,24 @@ inline int pool_tile_px(int C) {
     return p2;
 }
 
-// Slot (uint4 units) of entries (2*i2, 2*i2+1) of expert el in a mixing table
-// {row offset, row offset, weight, weight}: the four groups of a warp mix
-// experts 16 apart, so block b of 16 experts is shifted by b slots and their
-// reads hit different banks.
-__host__ __device__ __forceinline__ int pslot(int el, int kp, int i2) {
-    return el * (kp >> 1) + (el >> 4) + i2;
-}
-__host__ __device__ inline int pslot_count(int R, int kp) { return (R - 1) * (kp >> 1) + ((R - 1) >> 4) + (kp >> 1); }
-
-// Positions per tile of the two-pass path (moce_ring.cu).
-constexpr int kRingTile = 64;
+// Positions per tile of the stream path (moce_stream.cu).
+constexpr int kStreamTile = 64;
 
 struct WsLayout {
     size_t ctrl = 0;      // kCtrlWords uint32
-    size_t partial = 0;   // [N][pool_tiles][C] pooling tile sums: fp32 (multi-kernel path) or
-                          // tagged 64-bit words {fp32 bits, epoch + 1} (persistent kernels);
-                          // [N][ceil(HW/64)][C] tagged fp32 tile sums beyond the fixed-point
-                          // range (two-pass path)
+    size_t partial = 0;   // [N][pool_tiles][C] fp32 pooling tile sums (step kernels);
+                          // [N][ceil(HW/64)][C] tagged 64-bit words {fp32 bits, epoch + 1}:
+                          // tile sums beyond the fixed-point range (stream path)
     size_t z = 0;         // [N][C] fp32
     size_t tau = 0;       // [N][R] fp32
-    size_t a = 0;         // [N][R][k] mixing weights: fp32 (multi-kernel path) or tagged 64-bit;
-                          // softmax weight pairs in mixing-table order (two-pass path)
-    size_t zacc = 0;      // [N][4][C] int64 fixed-point channel sums (two-pass path)
-    size_t sync = 0;      // [2][N] uint32: tile arrivals, then the tag (epoch + 1) of the
-                          // forward that produced example n's weights (two-pass and stream paths)
+    size_t a = 0;         // [N][R][k] fp32 mixing weights (step kernels)
+    size_t zacc = 0;      // [2][N][C] 64-bit channel accumulator words (stream path)
+    size_t sync = 0;      // [2][N] uint32; [N + n]: the tag (epoch + 1) of the forward that
+                          // produced example n's weights (stream path)
     size_t sblk = 0;      // [N] weight blocks of the stream path (stream_table_bytes(R) each)
     size_t total = 0;
     int pool_px = 0;
     int pool_tiles = 0;
-    int gate_blocks = 0;
 };
 
 // Bytes of one example's weight block on the stream path: 16 floats per
@@ -79,20 +65,16 @@ inline WsLayout ws_layout(int N, int HW, int C, int R, int k) {
     WsLayout L;
     L.pool_px = pool_tile_px(C);
     L.pool_tiles = (HW + L.pool_px - 1) / L.pool_px;
-    L.gate_blocks = (R + kGateExperts - 1) / kGateExperts;
-    const size_t ring_tiles = (size_t)(HW + kRingTile - 1) / kRingTile;
-    const int kp = k + (k & 1);
+    const size_t stream_tiles = (size_t)(HW + kStreamTile - 1) / kStreamTile;
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     auto mx = [](size_t a, size_t b) { return a > b ? a : b; };
     L.ctrl = take(kCtrlWords * 4);
-    L.partial = take((size_t)N * mx((size_t)L.pool_tiles * C * 8, ring_tiles * C * 8));
+    L.partial = take((size_t)N * mx((size_t)L.pool_tiles * C * 4, stream_tiles * C * 8));
     L.z = take((size_t)N * C * 4);
     L.tau = take((size_t)N * R * 4);
-    // two-pass path: a 4 KB weight block per example ([32 pairs][8] float4)
-    (void)kp;
-    L.a = take((size_t)N * mx((size_t)R * k * 8, (size_t)4096));
-    L.zacc = take((size_t)N * 4 * C * 8);
+    L.a = take((size_t)N * R * k * 4);
+    L.zacc = take((size_t)2 * N * C * 8);
     L.sync = take((size_t)N * 8);
     L.sblk = take((size_t)N * stream_table_bytes(R));
     L.total = off;
@@ -144,33 +126,17 @@ cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_
                         const float *b2, float tmin, float tmax, float *tau, float *a,
                         cudaStream_t s);
 
+// ctrl: the workspace control words (bounded waits report MOCE_ERR_TIMEOUT there).
 cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
                        moce_layout_t lay, const int32_t *pidx, const float *a,
-                       const int32_t *resid, int nU, void *y, cudaStream_t s);
+                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s);
 
-cudaError_t launch_fused(const uint16_t *x, int N, int HW, int C, int R, int k,
-                         const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
-                         const float *W1, const float *b1, const float *w2, const float *b2,
-                         float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
-                         cudaStream_t s);
-
-bool fused_supported(int N, int HW, int C, int R, int k);
-
-cudaError_t launch_pipe(const uint16_t *x, int N, int HW, int C, int R, int k,
-                        const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
-                        const float *W1, const float *b1, const float *w2, const float *b2,
-                        float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
-                        cudaStream_t s);
-
-bool pipe_supported(int N, int HW, int C, int R, int k);
-
-cudaError_t launch_ring(const uint16_t *x, int N, int HW, int C, int R, int k,
-                        const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
-                        const float *W1, const float *b1, const float *w2, const float *b2,
-                        float tmin, float tmax, uint16_t *y, const WsLayout &L, unsigned char *ws,
-                        bool fused, cudaStream_t s);
-
-bool ring_supported(int N, int HW, int C, int R, int k, bool fused);
+// Mixing kernel for wide layers (moce_mix_wide.cu): NHWC bf16, C % 8 == 0,
+// x 16-byte aligned.
+bool mix_wide_supported(int HW, int C, int R, int k, int nU);
+cudaError_t launch_mix_wide(const uint16_t *x, int N, int HW, int C, int R, int k,
+                            const int32_t *pidx, const float *a, const int32_t *resid, int nU,
+                            uint16_t *y, uint32_t *ctrl, cudaStream_t s);
 
 cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
                           const int32_t *pidx, const float *plog, const int32_t *resid, int nU,

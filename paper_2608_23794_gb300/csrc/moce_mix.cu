@@ -4,13 +4,14 @@
 // The weights a[n,e,i] come from the gate stage. fp32 accumulation, output
 // rounded to the input dtype (bf16: round to nearest even).
 //
-// Three kernels:
+// NHWC bf16 with C % 8 == 0, k % 8 == 0 and aligned tables goes to
+// mix_wide_kernel (moce_mix_wide.cu); here:
 //  * mix_nchw_kernel: one thread per position, channel planes are contiguous
 //    so a warp's gathered loads are coalesced; any dtype.
 //  * mix_nhwc_generic_kernel: one thread per output element, for NHWC inputs
-//    the tiled kernel does not take (fp32, C % 8 != 0, unaligned x).
-//  * mix_nhwc_bf16_tile (device function, used by the tiled kernel and the
-//    fused persistent kernel): a tile of TP = 8*GS positions of one example is
+//    the tiled kernels do not take (fp32, C % 8 != 0, unaligned x).
+//  * mix_nhwc_bf16_tile (device function of the tiled kernel, for the other
+//    NHWC bf16 shapes): a tile of TP = 8*GS positions of one example is
 //    staged in shared memory transposed to channel-major rows (pixel pairs
 //    packed in 32-bit words, rows XOR-swizzled in 16-byte chunks so both the
 //    staging stores and the gathers are bank-conflict free); each group of GS
@@ -154,7 +155,7 @@ bool mix_geometry(int C, int R, int k, size_t budget, MixGeom *out) {
 
 cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
                        moce_layout_t lay, const int32_t *pidx, const float *a,
-                       const int32_t *resid, int nU, void *y, cudaStream_t s) {
+                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s) {
     if (N == 0 || HW == 0) return cudaSuccess;
     if (lay == MOCE_NCHW) {
         const int EPB = 8;
@@ -168,6 +169,11 @@ cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_d
                                                               resid, nU, EPB, (float *)y);
         return cudaGetLastError();
     }
+    if (dt == MOCE_BF16 && C % 8 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(pidx) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(a) & 15u) == 0 && mix_wide_supported(HW, C, R, k, nU))
+        return launch_mix_wide((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU,
+                               (uint16_t *)y, ctrl, s);
     MixGeom g;
     const bool tiled = dt == MOCE_BF16 && C % 8 == 0 &&
                        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&

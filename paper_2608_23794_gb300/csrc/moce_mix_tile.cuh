@@ -1,6 +1,6 @@
 // One tile of the NHWC bf16 routed mix + residual (Eq. (expert), Eq. (res)).
-// Used by the standalone tiled mixing kernel and by the fused persistent
-// forward kernel. See moce_mix.cu for the design notes.
+// Used by the standalone tiled mixing kernel (the shapes moce_mix_wide.cu
+// does not take). See moce_mix.cu for the design notes.
 #pragma once
 
 #include "moce_internal.cuh"

@@ -55,7 +55,7 @@ extern "C" moce_status_t moce_forward_noalloc(
     if (need > kNoAllocScratchBytes) return MOCE_ERR_UNSUPPORTED;
     void *scratch = nullptr;
     if (scratch_address(&scratch) != cudaSuccess) return MOCE_ERR_CUDA;
-    // The array keeps whatever the previous call left in it. The fused
+    // The array keeps whatever the previous call left in it. The stream
     // kernel's control words and tagged values must start from zero, so the
     // part this layer uses is cleared on the caller's stream first.
     if (cudaMemsetAsync(scratch, 0, need, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
@@ -63,4 +63,12 @@ extern "C" moce_status_t moce_forward_noalloc(
     return moce_forward(x, N, H, W, C_in, C_out, k, dtype, layout, packed_idx, packed_logits,
                         resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max, y, scratch, need,
                         stream);
+}
+
+// The control words sit at the start of the scratch (the workspace layout
+// every forward uses): the error word of the last forward on this device.
+extern "C" moce_status_t moce_noalloc_check_device_error(moce_stream_t stream) {
+    void *scratch = nullptr;
+    if (scratch_address(&scratch) != cudaSuccess) return MOCE_ERR_CUDA;
+    return moce_check_device_error(scratch, moce::kCtrlWords * 4, stream);
 }

@@ -69,6 +69,7 @@ def library():
             "moce_forward_launches": ([P, I, I, I, I, I, I, I, I], I),
             "moce_forward_kernel": ([P, I, I, I, I, I, I, I, I], ctypes.c_char_p),
             "moce_forward_noalloc": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P], I),
+            "moce_noalloc_check_device_error": ([P], I),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -213,7 +214,7 @@ def moce_gate(z: torch.Tensor, packed: PackedSupports, W1, b1, w2, b2, tau_min: 
 
 
 # moce_path_t: the kernel path of one forward (AUTO = the fastest that fits)
-PATHS = {"auto": 0, "pipe": 1, "two_pass": 2, "fused": 3, "steps": 4, "ring": 5, "stream": 6}
+PATHS = {"auto": 0, "steps": 4, "stream": 6}
 
 
 def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
@@ -288,6 +289,12 @@ def moce_forward_noalloc(x: torch.Tensor, layout: str, packed: PackedSupports, W
                                           float(tau_max), _ptr(y), _stream(stream)),
            "moce_forward_noalloc")
     return y
+
+
+def moce_noalloc_check_device_error(stream=None):
+    """Raise if a bounded wait of the last moce_forward_noalloc on this device gave up (synchronous)."""
+    _check(library().moce_noalloc_check_device_error(_stream(stream)),
+           "moce_noalloc_check_device_error")
 
 
 def moce_check_device_error(ws: Workspace, stream=None):

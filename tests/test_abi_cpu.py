@@ -106,30 +106,25 @@ def test_forward_path_selection_on_host(lib):
                  0.2, 6.0, fake, fake, ws_bytes, path, None)
 
     assert call(1, 7) == 1             # not a path
-    assert call(0, 5) == 3             # nor a single-pass ring kernel
+    for retired in (1, 2, 3, 5):       # values of kernels this library no longer has
+        assert call(1, retired) == 1
+        assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, retired) == 0
     assert call(1, -1) == 1
-    assert call(0, 2) == 3             # fp32 has no two-pass kernel: unsupported, nothing enqueued
-    assert call(0, 1) == 3             # nor a pipeline kernel
-    # bf16 NHWC, aligned x: every path runs these shapes
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 2   # the fastest: two-pass
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"moce_poolgate_kernel+moce_ring_kernel"
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 1) == b"moce_pipe_kernel"
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == 2
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 2) == b"moce_poolgate_kernel+moce_ring_kernel"
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 3) == 1
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 5) == 1
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 5) == b"moce_ring_kernel"
+    # without a GPU the stream kernel cannot be planned (no SM count, no
+    # tensor-map encoder): unsupported, nothing enqueued; AUTO takes the steps
+    assert call(1, 6) == 3
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 6) == 0
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 6) is None
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 4   # pool partials, pool, gate, mix
+    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"pool+gate+mix"
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
-    assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == b"pool+gate+mix"
-    # misaligned x or NCHW leaves only the step kernels
+    # fp32 has no stream kernel either; the steps run any dtype, layout and alignment
+    assert call(0, 6) == 3
     odd = ctypes.c_void_p(0x1002)
-    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 1) == 0
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 2) == 0
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3
-    # more experts than the two-pass kernel's pairs: the pipeline kernel
-    assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 2) == 0
-    assert n(fake, 2, 8, 8, 256, 96, 4, 1, 0, 1) == 1
-    assert name(fake, 2, 8, 8, 256, 96, 4, 1, 0, 0) == b"moce_pipe_kernel"
+    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 6) == 0
+    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 6) == 0
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3   # NCHW: pool, gate, mix
 
 
 def test_pack_rejects_bad_arguments_on_host(lib):

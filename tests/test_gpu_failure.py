@@ -1,13 +1,12 @@
 """Failure detection of the forward, without faulting the GPU.
 
 The fault is made on the host: the workspace's fault-injection word
-(scheduler word 4) names work item 0, the first pooling tile of example 0,
-which then computes but is never counted. On the two-pass path no CTA
-completes that example, so the mixing pass finds its weights missing; on the
-persistent kernels the bounded waits on that example run out. Either way the
-forward must exit, report MOCE_ERR_TIMEOUT through moce_check_device_error,
-leave the context usable, and a re-initialised workspace must give correct
-results.
+(control word 4) names work item 0, the first tile of example 0, whose
+channel sums are then computed but never added to the example's
+accumulator words. The stream kernel's gate for that example, and every
+wait on its weights, then runs out its bounded wait. The forward must exit,
+report MOCE_ERR_TIMEOUT through moce_check_device_error, leave the context
+usable, and a re-initialised workspace must give correct results.
 """
 import numpy as np
 import pytest
@@ -19,7 +18,7 @@ pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
 
 
-@pytest.mark.parametrize("path", ["stream", "pipe", "two_pass", "ring", "fused"])
+@pytest.mark.parametrize("path", ["stream"])
 def test_bounded_wait_reports_timeout_and_recovers(path):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
@@ -28,7 +27,7 @@ def test_bounded_wait_reports_timeout_and_recovers(path):
     cfg = synth.LayerConfig("fail", 4, 16, 16, 64, 16, 4, "bf16", "nhwc", "relu", 56)
     lay = synth.make_layer(cfg, seed=9)
     dev = device_tensors(lay)
-    assert moce.moce_forward_launches(dev["x"], "nhwc", cfg.C_out, cfg.k, path=path) in (1, 2)
+    assert moce.moce_forward_launches(dev["x"], "nhwc", cfg.C_out, cfg.k, path=path) == 1
     packed = moce.moce_pack_supports(dev["support_idx"], dev["support_logits"], cfg.C_in)
     ws = moce.Workspace(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k)
     run = lambda: moce.moce_forward(dev["x"], "nhwc", packed, dev["W1"], dev["b1"], dev["w2"],

@@ -3,20 +3,20 @@
 Such callers (allocator or pool callbacks, loops that forbid allocation after
 start-up, plugins whose framework owns every buffer) cannot provide a
 workspace; this entry point uses a fixed scratch array inside the library.
-Its output must match moce_forward on the same inputs, on consecutive calls
-that reuse the shared array. This file is named to run last.
+Its output must match moce_forward on the same inputs and the CPU oracle, on
+consecutive calls that reuse the shared array. This file is named to run last.
 """
 import numpy as np
 import pytest
 
-from moce_cases import TOL, device_tensors
+from moce_cases import TOL, assert_close, device_tensors, oracle_forward
 from paper_2608_23794_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
 
 CASES = [
-    synth.CONFIGS["rn50_stage1_reduce"].replace(N=8),           # fused kernel
+    synth.CONFIGS["rn50_stage1_reduce"].replace(N=8),           # stream kernel
     synth.CONFIGS["tiny_f32_nchw"],                             # multi-kernel path
     synth.LayerConfig("c72", 3, 9, 11, 72, 9, 5, "bf16", "nhwc", "gelu", 60),
 ]
@@ -35,11 +35,13 @@ def test_noalloc_matches_forward_on_two_calls(cfg):
     ref = moce.moce_forward(dev["x"], cfg.layout, packed, *args)
     ref = ref.float().cpu().numpy().astype(np.float64)
     tol = TOL[cfg.dtype]
+    yref = oracle_forward(lay)
     for _ in range(2):
         got = moce.moce_forward_noalloc(dev["x"], cfg.layout, packed, *args)
-        torch.cuda.synchronize()
+        moce.moce_noalloc_check_device_error()
         got = got.float().cpu().numpy().astype(np.float64)
         assert np.all(np.abs(got - ref) <= tol + tol * np.abs(ref))
+        assert_close(got, yref, cfg.dtype, "noalloc y")
 
 
 def test_noalloc_rejects_layers_beyond_its_scratch():
