@@ -28,7 +28,8 @@ __global__ void __launch_bounds__(kThreads) gate_kernel(
                tau, a);
 }
 
-constexpr int kTE = 64;  // experts per tiled-gate CTA
+constexpr int kTE = 64;        // experts per tiled-gate CTA
+constexpr int kUS = kTE + 4;   // padded row of U^T (float4-aligned, rows 4 banks apart)
 
 __host__ __device__ inline int tiled_kc(int k) {
     int kc = 24576 / k;  // W1^T chunk of at most 96 KB
@@ -36,13 +37,13 @@ __host__ __device__ inline int tiled_kc(int k) {
     return kc & ~3;
 }
 // Floats of the W1^T buffer, which first holds z of the example and the
-// CTA's block of support indices (C floats plus kTE k indices).
+// CTA's block of support indices (C floats plus kTE rows of k + 1 indices).
 __host__ __device__ inline size_t tiled_wt(int k, int C) {
-    const size_t a = (size_t)tiled_kc(k) * k, b = (size_t)C + (size_t)kTE * k;
+    const size_t a = (size_t)tiled_kc(k) * k, b = (size_t)C + (size_t)kTE * (k + 1);
     return a > b ? a : b;
 }
 __host__ __device__ inline size_t tiled_smem(int k, int C) {
-    return ((size_t)k * kTE + tiled_wt(k, C) + kTE) * sizeof(float);
+    return ((size_t)k * kUS + tiled_wt(k, C) + kTE) * sizeof(float);
 }
 
 template <int TN>
@@ -54,25 +55,33 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
     constexpr int k = 16 * TN;
     extern __shared__ __align__(16) float tsm[];
     const int KC = tiled_kc(k);
-    float *Ut = tsm;                      // [k][kTE]
-    float *Wt = Ut + (size_t)k * kTE;     // [KC][k]: Wt[i][j] = W1[j][i0 + i]
+    float *Ut = tsm;                      // [k][kUS]: Ut[i][el] = z[n, S_(e0 + el)][i]
+    float *Wt = Ut + (size_t)k * kUS;     // [KC][k]: Wt[i][j] = W1[j][i0 + i]
     float *tau_s = Wt + tiled_wt(k, C);   // [kTE]
     const int n = blockIdx.y, e0 = blockIdx.x * kTE;
     const int tid = threadIdx.x, te = tid >> 4, th = tid & 15;
     const float *zn = z + (size_t)n * C;
 
     {
-        // stage z_n and the block's support indices (coalesced), then gather
+        // stage z_n and the block's support indices (coalesced loads; index
+        // rows of k + 1 so that the gather below reads them without bank
+        // conflicts), then gather U^T with consecutive threads on consecutive
+        // experts (conflict-free stores)
         float *zs = Wt;
         int32_t *is = reinterpret_cast<int32_t *>(Wt + C);
         const int ne = min(kTE, R - e0);
         for (int c = tid; c < C; c += 256) zs[c] = __ldcg(zn + c);
         const int4 *src = reinterpret_cast<const int4 *>(pidx + (size_t)e0 * k);
-        for (int q = tid; q < ne * k / 4; q += 256) reinterpret_cast<int4 *>(is)[q] = __ldg(src + q);
+        for (int q = tid; q < ne * k / 4; q += 256) {
+            const int4 v = __ldg(src + q);
+            const int el = (4 * q) / k, i = 4 * q - el * k;
+            int32_t *d = is + (size_t)el * (k + 1) + i;
+            d[0] = v.x; d[1] = v.y; d[2] = v.z; d[3] = v.w;
+        }
         __syncthreads();
         for (int q = tid; q < kTE * k; q += 256) {
-            const int el = q / k, i = q - el * k;
-            Ut[i * kTE + el] = el < ne ? zs[is[q]] : 0.f;
+            const int el = q & (kTE - 1), i = q / kTE;
+            Ut[i * kUS + el] = el < ne ? zs[is[el * (k + 1) + i]] : 0.f;
         }
     }
     // thread th's hidden units, in pairs: pair p < 2 (TN / 4) is units
@@ -104,7 +113,7 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
         __syncthreads();
 #pragma unroll 2
         for (int i = 0; i < kc; ++i) {
-            const float4 u = *reinterpret_cast<const float4 *>(Ut + (size_t)(i0 + i) * kTE + 4 * te);
+            const float4 u = *reinterpret_cast<const float4 *>(Ut + (size_t)(i0 + i) * kUS + 4 * te);
             const float *wr = Wt + (size_t)i * k;
             float2 w[NP];
 #pragma unroll

@@ -325,9 +325,10 @@ bool wide_geometry(int HW, int C, int R, int k, int nU, WideGeom *out) {
         g.off_us = align_up(g.off_ys + (size_t)g.TP * YS * 2, 16);
         g.off_bar = align_up(g.off_us + (size_t)(nU > 0 ? nU : 1) * 2, 16);
         g.off_tab = align_up(g.off_bar + 64, 128);
-        // chunks of 16 EPW experts (every warp busy), halved until they fit
+        // chunks of 16 EPW experts (every warp busy), halved until they fit,
+        // down to 4 EPW (a quarter of the warps busy)
         bool fit = false;
-        for (int eb = 16 * g.EPW; eb >= 1 && !fit; eb /= 2) {
+        for (int eb = 16 * g.EPW; eb >= 4 * g.EPW && !fit; eb /= 2) {
             const int ebc = eb < R ? eb : R;
             for (int nb = 3; nb >= 2 && !fit; --nb) {
                 const size_t sm = g.off_tab + (size_t)nb * 2 * ebc * k * 4;
