@@ -65,8 +65,9 @@ def _load():
                                             P, P, P, P]
         lib.moce_oracle_bruteforce_forward.argtypes = [P, I, I, I, I, I, I, I, P, P, P, P, F, D, D,
                                                        P]
+        lib.moce_oracle_coverage.argtypes = [I, I, P, D, P, P, P]
         for fn in (lib.moce_oracle_topk, lib.moce_oracle_pack, lib.moce_oracle_forward,
-                   lib.moce_oracle_bruteforce_forward):
+                   lib.moce_oracle_bruteforce_forward, lib.moce_oracle_coverage):
             fn.restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -96,6 +97,22 @@ def topk(L: np.ndarray, k: int):
     if st != OK:
         raise OracleError(st, "topk")
     return idx, lg
+
+
+def coverage(L: np.ndarray, eps: float, grad: bool = True):
+    """Sec. 3.4 coverage regularizer over the full routing matrix L [R, C].
+
+    Returns (loss, u [C], dloss/dL [R, C] or None), all float64.
+    """
+    L = _c(L, np.float32)
+    R, C = L.shape
+    loss = np.zeros(1, np.float64)
+    u = np.empty(C, np.float64)
+    g = np.empty((R, C), np.float64) if grad else None
+    st = _load().moce_oracle_coverage(C, R, _p(L), float(eps), _p(loss), _p(u), _p(g))
+    if st != OK:
+        raise OracleError(st, "coverage")
+    return float(loss[0]), u, g
 
 
 def pack(support_idx: np.ndarray, support_logits: np.ndarray, C: int):
@@ -244,7 +261,7 @@ class _use_library:
         # reuse the argtypes of the real build
         for name in ("moce_oracle_topk", "moce_oracle_pack", "moce_oracle_pool", "moce_oracle_gate",
                      "moce_oracle_weights", "moce_oracle_mix", "moce_oracle_forward",
-                     "moce_oracle_bruteforce_forward"):
+                     "moce_oracle_bruteforce_forward", "moce_oracle_coverage"):
             src, dst = getattr(self._saved, name), getattr(lib, name)
             dst.argtypes, dst.restype = src.argtypes, src.restype
         _lib = lib

@@ -20,6 +20,8 @@
  *   weights   Eq. (weights)                 a = softmax(L_S / tau)
  *   routed    Eq. (expert)                  Y_e = sum_i a_i X_i
  *   residual  Eq. (res), Sec. 3.4           mean of X over U, 0 if U is empty
+ *   coverage  Sec. 3.4                      L_cov over the full routing matrix and
+ *             its gradient with respect to every logit (chain rule, written out)
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - ties between equal logits order by ascending channel index; -0.0 and
@@ -28,7 +30,8 @@
  *     g = w2 . h + b2, sigma is the logistic function;
  *   - the softmax subtracts the largest support logit before exponentiating,
  *     which leaves Eq. (weights) unchanged;
- *   - U is listed in ascending channel order.
+ *   - U is listed in ascending channel order;
+ *   - the coverage loss's epsilon is an argument (the paper does not print it).
  *
  * Inputs are the exact values the device sees (bf16 inputs are decoded to
  * float first); all arithmetic is in double.
@@ -395,5 +398,87 @@ int moce_oracle_bruteforce_forward(const float *x, int N, int H, int W, int C, i
             }
     }
     free(sel); free(count); free(taken); free(Weff); free(zn); free(hid);
+    return ORACLE_OK;
+}
+
+/*
+ * Coverage regularizer, Sec. 3.4: p_{e,c} = softmax(L_e)_c over all C
+ * channels of a full routing row, u_c = (1/R) sum_e p_{e,c},
+ * ubar = (1/C) sum_c u_c, L_cov = sum_c (u_c - ubar)^2 / (ubar^2 + eps).
+ * L is [R][C]. Writes the loss; u [C] and the gradient dL_cov/dL [R][C] when
+ * the pointers are not NULL. The softmax subtracts the row maximum first.
+ * The gradient is the chain rule of the same definitions:
+ *   dL/du_c = 2 (u_c - ubar) / D - (2 / C) sum_c' (u_c' - ubar) / D
+ *             - 2 ubar S / (C D^2),     D = ubar^2 + eps, S = sum_c (u_c - ubar)^2
+ *   dL/dL_{e,c} = (1/R) p_{e,c} (dL/du_c - sum_c' p_{e,c'} dL/du_c').
+ */
+int moce_oracle_coverage(int C, int R, const float *L, double eps, double *loss, double *u_out,
+                         double *grad)
+{
+    if (C < 1 || R < 1 || !L || !loss || !(eps >= 0.0))
+        return ORACLE_BAD_ARG;
+    double *p = (double *)malloc(sizeof(double) * (size_t)R * C);
+    double *u = (double *)malloc(sizeof(double) * (size_t)C);
+    double *g = (double *)malloc(sizeof(double) * (size_t)C);
+    if (!p || !u || !g) {
+        free(p);
+        free(u);
+        free(g);
+        return ORACLE_NO_MEMORY;
+    }
+    for (int e = 0; e < R; ++e) {
+        const float *Le = L + (size_t)e * C;
+        double m = -INFINITY;
+        for (int c = 0; c < C; ++c) {
+            if (!isfinite(Le[c])) {
+                free(p);
+                free(u);
+                free(g);
+                return ORACLE_BAD_SUPPORT;
+            }
+            if ((double)Le[c] > m)
+                m = (double)Le[c];
+        }
+        double sum = 0.0;
+        for (int c = 0; c < C; ++c)
+            sum += exp((double)Le[c] - m);
+        for (int c = 0; c < C; ++c)
+            p[(size_t)e * C + c] = exp((double)Le[c] - m) / sum;
+    }
+    for (int c = 0; c < C; ++c) {
+        double s = 0.0;
+        for (int e = 0; e < R; ++e)
+            s += p[(size_t)e * C + c];
+        u[c] = s / (double)R;
+    }
+    double ubar = 0.0;
+    for (int c = 0; c < C; ++c)
+        ubar += u[c];
+    ubar /= (double)C;
+    const double D = ubar * ubar + eps;
+    double S = 0.0, dev = 0.0;
+    for (int c = 0; c < C; ++c) {
+        S += (u[c] - ubar) * (u[c] - ubar);
+        dev += u[c] - ubar;
+    }
+    *loss = S / D;
+    if (u_out)
+        for (int c = 0; c < C; ++c)
+            u_out[c] = u[c];
+    if (grad) {
+        for (int c = 0; c < C; ++c)
+            g[c] = 2.0 * (u[c] - ubar) / D - 2.0 * dev / ((double)C * D) -
+                   2.0 * ubar * S / ((double)C * D * D);
+        for (int e = 0; e < R; ++e) {
+            double dot = 0.0;
+            for (int c = 0; c < C; ++c)
+                dot += p[(size_t)e * C + c] * g[c];
+            for (int c = 0; c < C; ++c)
+                grad[(size_t)e * C + c] = p[(size_t)e * C + c] * (g[c] - dot) / (double)R;
+        }
+    }
+    free(p);
+    free(u);
+    free(g);
     return ORACLE_OK;
 }

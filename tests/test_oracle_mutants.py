@@ -39,6 +39,16 @@ MUTANTS = {
     "pack_ties_descending_index": ("return (a->idx > b->idx) - (a->idx < b->idx);",
                                    "return (a->idx < b->idx) - (a->idx > b->idx);"),
     "pack_no_duplicate_check": ("seen_in_row[c] == e", "0"),
+    "coverage_softmax_over_experts": ("        for (int c = 0; c < C; ++c)\n            sum += exp((double)Le[c] - m);",
+                                      "        for (int c = 0; c < C; ++c)\n            sum += exp((double)Le[c] - m) * (double)R / (double)C;"),
+    "coverage_u_not_averaged": ("u[c] = s / (double)R;", "u[c] = s;"),
+    "coverage_no_eps": ("const double D = ubar * ubar + eps;", "const double D = ubar * ubar;"),
+    # (a term that is the same for every channel cancels in dL/dL through the
+    # softmax Jacobian, so dropping one is not a mistake; flipping the
+    # per-channel deviation is)
+    "coverage_grad_deviation_sign": ("g[c] = 2.0 * (u[c] - ubar) / D", "g[c] = 2.0 * (ubar - u[c]) / D"),
+    "coverage_grad_softmax_jacobian_dot_dropped": ("p[(size_t)e * C + c] * (g[c] - dot) / (double)R;",
+                                                   "p[(size_t)e * C + c] * g[c] / (double)R;"),
 }
 
 PIN_CHECKS = [
@@ -59,6 +69,10 @@ PIN_CHECKS = [
     pins.test_empty_residual_is_exactly_zero,
     lambda: pins.test_forward_equals_bruteforce("nhwc", 0),
     pins.test_fixed_temperature_is_a_linear_map,
+    pins.test_coverage_uniform_rows_are_zero,
+    lambda: pins.test_coverage_one_expert_two_channels_closed_form(2.5, -1.0),
+    pins.test_coverage_row_shift_and_channel_permutation,
+    pins.test_coverage_equals_numpy_definition_and_finite_differences,
 ]
 
 

@@ -120,6 +120,85 @@ def test_topk_equals_stable_argsort():
     assert lg.tolist() == np.take_along_axis(L, ref, 1).tolist()
 
 
+# ---------------------------------------------------------------- coverage (Sec. 3.4)
+
+
+def test_coverage_uniform_rows_are_zero():
+    # equal logits in every row: p = 1/C, u = 1/C = ubar, so L_cov = 0 and dL_cov/dL = 0
+    L = np.full((5, 12), 0.7, np.float32)
+    loss, u, g = oracle.coverage(L, 1e-8)
+    assert loss == 0.0
+    np.testing.assert_allclose(u, 1.0 / 12, rtol=0, atol=1e-15)
+    np.testing.assert_allclose(g, 0.0, atol=1e-12)
+
+
+@pytest.mark.parametrize("a,b", [(0.0, 1.0), (2.5, -1.0), (-0.3, -0.3)])
+def test_coverage_one_expert_two_channels_closed_form(a, b):
+    # R = 1, C = 2: p = (s, 1 - s), s = 1 / (1 + exp(b - a)); ubar = 1/2, so
+    # L_cov = 2 (s - 1/2)^2 / (1/4 + eps); dL_cov/da = 4 (s - 1/2) s (1 - s) / (1/4 + eps)
+    eps = 1e-3
+    s = 1.0 / (1.0 + math.exp(float(np.float32(b)) - float(np.float32(a))))
+    loss, u, g = oracle.coverage(np.array([[a, b]], np.float32), eps)
+    assert loss == pytest.approx(2 * (s - 0.5) ** 2 / (0.25 + eps), rel=1e-12, abs=1e-15)
+    np.testing.assert_allclose(u, [s, 1 - s], rtol=1e-12)
+    da = 4 * (s - 0.5) * s * (1 - s) / (0.25 + eps)
+    np.testing.assert_allclose(g[0], [da, -da], rtol=1e-9, atol=1e-15)
+
+
+def test_coverage_row_shift_and_channel_permutation():
+    rng = np.random.default_rng(4)
+    L = rng.standard_normal((6, 9)).astype(np.float32)
+    loss, _, g = oracle.coverage(L, 1e-6)
+    # a constant added to one row leaves its softmax unchanged
+    L2 = L.copy()
+    L2[2] += np.float32(1.5)
+    loss2, _, g2 = oracle.coverage(L2, 1e-6)
+    assert loss2 == pytest.approx(loss, rel=1e-6)
+    np.testing.assert_allclose(g2, g, rtol=1e-5, atol=1e-9)
+    # permuting the channels of every row permutes u and the gradient
+    perm = rng.permutation(9)
+    loss3, _, g3 = oracle.coverage(L[:, perm], 1e-6)
+    assert loss3 == pytest.approx(loss, rel=1e-12)
+    np.testing.assert_allclose(g3, g[:, perm], rtol=1e-10, atol=1e-14)
+
+
+def test_coverage_equals_numpy_definition_and_finite_differences():
+    rng = np.random.default_rng(8)
+    L = (1.7 * rng.standard_normal((4, 7))).astype(np.float32)
+    eps = 1e-2
+    loss, u, g = oracle.coverage(L, eps)
+    # the definition with scipy's softmax over the channel axis
+    P = sp_softmax(L.astype(np.float64), axis=1)
+    uu = P.mean(axis=0)
+    assert loss == pytest.approx(((uu - uu.mean()) ** 2).sum() / (uu.mean() ** 2 + eps), rel=1e-12)
+    np.testing.assert_allclose(u, uu, rtol=1e-12)
+
+    # central differences of the same definition in float64
+    def f(Ld):
+        Pd = sp_softmax(Ld, axis=1)
+        ud = Pd.mean(axis=0)
+        return ((ud - ud.mean()) ** 2).sum() / (ud.mean() ** 2 + eps)
+
+    h = 1e-6
+    fd = np.zeros_like(g)
+    for e in range(L.shape[0]):
+        for c in range(L.shape[1]):
+            Lp, Lm = L.astype(np.float64), L.astype(np.float64)
+            Lp[e, c] += h
+            Lm[e, c] -= h
+            fd[e, c] = (f(Lp) - f(Lm)) / (2 * h)
+    np.testing.assert_allclose(g, fd, rtol=1e-6, atol=1e-10)
+    assert abs(g.sum()) < 1e-12  # a common shift of all logits changes nothing
+
+
+def test_coverage_rejects_non_finite():
+    L = np.zeros((2, 3), np.float32)
+    L[1, 2] = np.inf
+    with pytest.raises(oracle.OracleError) as ei:
+        oracle.coverage(L, 1e-8)
+    assert ei.value.status == oracle.BAD_SUPPORT
+
+
 # ---------------------------------------------------------------- pooling
 
 
