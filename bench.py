@@ -54,6 +54,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto",
                     help="kernel path of the forward (auto, stream, steps)")
+    ap.add_argument("--op", choices=["forward", "train"], default="forward",
+                    help="forward: the layer forward (the benchmark); train: TopK over the full "
+                         "routing matrix and the coverage loss with its gradient")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline leg")
     return ap.parse_args()
@@ -539,10 +542,77 @@ def run_ours(args, cfg):
         torch.distributed.destroy_process_group()
 
 
+def run_train(args, cfg):
+    """Support maintenance on the layer's routing matrix L [C_out, C_in] (Sec. 3.2 TopK, Sec. 3.4
+    coverage loss and gradient): device time per call, GB/s of the algorithmic bytes, and the
+    oracle on one host core beside it."""
+    import numpy as np
+    import torch
+
+    from paper_2608_23794_gb300 import build as moce_build
+    from paper_2608_23794_gb300 import moce
+
+    torch.cuda.set_device(0)
+    moce_build.build()
+    R, C, k = cfg.C_out, cfg.C_in, cfg.k
+    rng = np.random.default_rng(SEED)
+    L = rng.standard_normal((R, C)).astype(np.float32)
+    dL = torch.from_numpy(L).cuda()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, reps):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / reps
+
+    reps = max(10, min(args.steps, 2000))
+    topk_us = timed(lambda: moce.moce_topk_supports(dL, k), reps)
+    cov_us = timed(lambda: moce.moce_coverage_loss(dL, 1e-8), reps)
+    cov_nograd_us = timed(lambda: moce.moce_coverage_loss(dL, 1e-8, grad=False), reps)
+    topk_bytes = R * C * 4 + R * k * 8
+    cov_bytes = 2 * R * C * 4  # L read once, the gradient written once
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        t0 = time.perf_counter()
+        oracle.topk(L, k)
+        t1 = time.perf_counter()
+        oracle.coverage(L, 1e-8)
+        t2 = time.perf_counter()
+        cpu = {"topk_us": (t1 - t0) * 1e6, "coverage_us": (t2 - t1) * 1e6, "cores": 1,
+               "kind": "oracle", "sample": f"the whole {R} x {C} routing matrix, one run"}
+    peaks, _ = measured_peaks()
+    line = {"metric": "MoCE support maintenance: TopK over the routing matrix + coverage loss and "
+                      "gradient (µs per call, GB/s of algorithmic bytes)",
+            "value": cov_bytes / cov_us / 1e3, "unit": UNIT, "n_gpus": 1, "steps": reps,
+            "warmup": args.warmup, "higher_is_better": True, "dtype": "f32",
+            "data": "synthetic (seeded N(0,1) routing logits)",
+            "config": {"workload": cfg.name, "C_out": R, "C_in": C, "k": k, "op": "train"},
+            "topk": {"us": topk_us, "GB/s": topk_bytes / topk_us / 1e3,
+                     "note": "the call is synchronous (it validates): device time between events "
+                             "includes the error-word copy"},
+            "coverage_with_grad": {"us": cov_us, "GB/s": cov_bytes / cov_us / 1e3,
+                                   "frac_of_hbm": cov_bytes / cov_us / 1e3 / peaks["hbm_gbs"]},
+            "coverage_loss_only": {"us": cov_nograd_us},
+            "gpu_launches": 6 * reps,
+            "cpu_baseline": cpu}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     from paper_2608_23794_gb300 import synth
     cfg = synth.CONFIGS[args.workload]
+    if args.op == "train":
+        run_train(args, cfg)
+        return
     if args.impl == "ours" and (cfg.dtype, cfg.layout) != ("bf16", "nhwc"):
         raise SystemExit(f"bench.py times bf16 NHWC layers; {cfg.name} is {cfg.dtype} {cfg.layout}")
     if args.impl == "reference":

@@ -273,6 +273,48 @@ const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_i
                                      moce_path_t path);
 
 /*
+ * Support maintenance on the full routing matrix (training side; the forward
+ * uses packed, fixed supports). logits: device fp32 [C_out][C_in], row e =
+ * L_e, the routing preferences of routed expert e over every input channel.
+ *
+ * Bytes of device workspace moce_topk_supports and moce_coverage_loss need
+ * (256-byte aligned; contents need no initialisation). 0 for invalid shapes.
+ */
+size_t moce_train_workspace_bytes(int C_in, int C_out);
+
+/*
+ * Eq. (support), Sec. 3.2: S_e = TopK(L_e, k) for every routed expert,
+ * written directly in deployment order (descending logit, equal logits by
+ * ascending channel, -0.0 equal to +0.0), i.e. as moce_pack_supports would
+ * order them:
+ *   packed_idx    device int32 [C_out][k] out: the selected channels
+ *   packed_logits device fp32 [C_out][k] out: their logits
+ * SYNCHRONOUS (it validates): a non-finite logit returns
+ * MOCE_ERR_BAD_SUPPORT (outputs then unspecified). C_in up to 16384
+ * (MOCE_ERR_UNSUPPORTED beyond: one CTA sorts a row in shared memory).
+ */
+moce_status_t moce_topk_supports(const float *logits, int C_in, int C_out, int k,
+                                 int32_t *packed_idx, float *packed_logits, void *ws,
+                                 size_t ws_bytes, moce_stream_t stream);
+
+/*
+ * The coverage regularizer of Sec. 3.4 over the full routing matrix:
+ *   p_{e,c} = softmax(L_e)_c over all C_in channels, u_c = (1/C_out) sum_e p_{e,c},
+ *   ubar = (1/C_in) sum_c u_c, L_cov = sum_c (u_c - ubar)^2 / (ubar^2 + eps).
+ *   loss  device fp32 [1] out: L_cov
+ *   usage device fp32 [C_in] out: u, or NULL
+ *   grad  device fp32 [C_out][C_in] out: dL_cov / dL, or NULL (the gradient
+ *         reaches every logit, selected or not, Sec. 3.2)
+ * eps >= 0 (the paper does not print its value). Sums run in a fixed order
+ * (u, ubar and the loss in double): results do not depend on scheduling.
+ * Asynchronous; logits are not validated (a non-finite logit gives a
+ * non-finite loss).
+ */
+moce_status_t moce_coverage_loss(const float *logits, int C_in, int C_out, float eps,
+                                 float *loss, float *usage, float *grad, void *ws,
+                                 size_t ws_bytes, moce_stream_t stream);
+
+/*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word the
  * forward kernels leave in `ws` (a forward workspace). Returns MOCE_OK,
  * MOCE_ERR_TIMEOUT (a bounded inter-CTA wait gave up; outputs of that call

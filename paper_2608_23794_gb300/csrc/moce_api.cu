@@ -238,6 +238,44 @@ const char *moce_forward_path_kernel(const void *x, int N, int H, int W, int C_i
     }
 }
 
+size_t moce_train_workspace_bytes(int C_in, int C_out) {
+    if (!shape_ok(0, 0, 0, C_in, C_out, 1)) return 0;
+    return train_ws_bytes(C_out, C_in);
+}
+
+moce_status_t moce_topk_supports(const float *logits, int C_in, int C_out, int k,
+                                 int32_t *packed_idx, float *packed_logits, void *ws,
+                                 size_t ws_bytes, moce_stream_t stream) {
+    if (!shape_ok(0, 0, 0, C_in, C_out, k)) return MOCE_ERR_INVALID_VALUE;
+    if (!logits || !packed_idx || !packed_logits || !ws) return MOCE_ERR_INVALID_VALUE;
+    if (ws_bytes < train_ws_bytes(C_out, C_in) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MOCE_ERR_INVALID_VALUE;
+    if ((size_t)topk_padded(C_in) * 8 > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t *err_word = static_cast<uint32_t *>(ws);
+    cudaError_t err = cudaMemsetAsync(err_word, 0, 4, s);
+    if (err == cudaSuccess)
+        err = launch_topk(logits, C_out, C_in, k, packed_idx, packed_logits, err_word, s);
+    uint32_t flag = 0;
+    if (err == cudaSuccess) err = cudaMemcpyAsync(&flag, err_word, 4, cudaMemcpyDeviceToHost, s);
+    if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+    if (err != cudaSuccess) return MOCE_ERR_CUDA;
+    return flag ? MOCE_ERR_BAD_SUPPORT : MOCE_OK;
+}
+
+moce_status_t moce_coverage_loss(const float *logits, int C_in, int C_out, float eps,
+                                 float *loss, float *usage, float *grad, void *ws,
+                                 size_t ws_bytes, moce_stream_t stream) {
+    if (!shape_ok(0, 0, 0, C_in, C_out, 1) || !(eps >= 0.f) || !isfinite(eps))
+        return MOCE_ERR_INVALID_VALUE;
+    if (!logits || !loss || !ws) return MOCE_ERR_INVALID_VALUE;
+    if (ws_bytes < train_ws_bytes(C_out, C_in) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MOCE_ERR_INVALID_VALUE;
+    return cuda_status(launch_coverage(logits, C_out, C_in, (double)eps, loss, usage, grad,
+                                       static_cast<unsigned char *>(ws),
+                                       reinterpret_cast<cudaStream_t>(stream)));
+}
+
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {
     if (!ws || ws_bytes < kCtrlWords * 4) return MOCE_ERR_INVALID_VALUE;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

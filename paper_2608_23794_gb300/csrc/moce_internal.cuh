@@ -138,6 +138,15 @@ cudaError_t launch_mix_wide(const uint16_t *x, int N, int HW, int C, int R, int 
                             const int32_t *pidx, const float *a, const int32_t *resid, int nU,
                             uint16_t *y, uint32_t *ctrl, cudaStream_t s);
 
+// Support maintenance (moce_train.cu): TopK over full routing rows and the
+// coverage regularizer.
+int topk_padded(int C);
+size_t train_ws_bytes(int R, int C);
+cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float *lg,
+                        uint32_t *err, cudaStream_t s);
+cudaError_t launch_coverage(const float *L, int R, int C, double eps, float *loss, float *u,
+                            float *grad, unsigned char *ws, cudaStream_t s);
+
 cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
                           const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
                           const float *W1, const float *b1, const float *w2, const float *b2,

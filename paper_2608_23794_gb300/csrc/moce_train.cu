@@ -1,0 +1,251 @@
+// Support maintenance on the full routing matrix L [R][C] (training side):
+//
+//   topk_rows_kernel      Eq. (support), Sec. 3.2: S_e = TopK(L_e, k), written in
+//                         deployment order (descending logit, equal logits by
+//                         ascending channel; -0.0 equals +0.0), so the result
+//                         is already packed. One CTA per expert row: the row's
+//                         C (key, channel) pairs are sorted in shared memory by
+//                         a bitonic network on 64-bit keys whose high word
+//                         orders the logit and whose low word is the channel.
+//   coverage kernels      Sec. 3.4: p_{e,c} = softmax(L_e)_c over all C channels,
+//                         u_c = (1/R) sum_e p_{e,c}, ubar = (1/C) sum_c u_c,
+//                         L_cov = sum_c (u_c - ubar)^2 / (ubar^2 + eps), and
+//                         dL_cov/dL_{e,c} = (1/R) p_{e,c} (g_c - sum_c' p_{e,c'} g_c')
+//                         with g_c = dL_cov/du_c. Row statistics (max, sum of
+//                         exponentials), then partial column sums over chunks
+//                         of kRowChunk rows (in row order, in double), then u
+//                         (the chunks in order), then the loss and g (one CTA,
+//                         double), then the gradient by rows.
+// Every sum runs in a fixed order: the results do not depend on scheduling.
+#include <math.h>
+
+#include "moce_internal.cuh"
+
+namespace moce {
+namespace {
+
+constexpr int kTrainThreads = 512;
+constexpr int kRowChunk = 32;  // rows per partial column sum
+constexpr uint32_t kTopkBadLogit = 1u;
+
+// Order key of a logit: larger logit -> smaller key; -0.0 and +0.0 equal.
+__device__ __forceinline__ uint32_t desc_key(float v) {
+    uint32_t b = __float_as_uint(v == 0.f ? 0.f : v);
+    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);  // increasing with v
+    return ~b;
+}
+
+__device__ float block_sum_f(float v, float *red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    float s = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];  // warp order
+    return s;
+}
+__device__ float block_max_f(float v, float *red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    float s = -INFINITY;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s = fmaxf(s, red[w]);
+    return s;
+}
+__device__ double block_sum_d(double v, double *red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    double s = 0.0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
+    return s;
+}
+
+// One expert row: CP = C rounded up to a power of two keys in shared memory.
+__global__ void __launch_bounds__(kTrainThreads) topk_rows_kernel(const float *__restrict__ L,
+                                                                   int C, int CP, int k,
+                                                                   int32_t *__restrict__ idx_out,
+                                                                   float *__restrict__ lg_out,
+                                                                   uint32_t *err) {
+    extern __shared__ unsigned long long keys[];
+    const int e = blockIdx.x;
+    const float *Le = L + (size_t)e * C;
+    for (int c = threadIdx.x; c < CP; c += kTrainThreads) {
+        unsigned long long key = ~0ull;
+        if (c < C) {
+            const float v = Le[c];
+            if (!isfinite(v)) atomicOr(err, kTopkBadLogit);
+            key = ((unsigned long long)desc_key(v) << 32) | (uint32_t)c;
+        }
+        keys[c] = key;
+    }
+    __syncthreads();
+    // bitonic sort, ascending keys
+    for (int size = 2; size <= CP; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = threadIdx.x; i < CP / 2; i += kTrainThreads) {
+                const int lo = 2 * i - (i & (stride - 1));  // pair (lo, lo + stride)
+                const int hi = lo + stride;
+                const bool up = (lo & size) == 0;
+                const unsigned long long a = keys[lo], b = keys[hi];
+                if ((a > b) == up) {
+                    keys[lo] = b;
+                    keys[hi] = a;
+                }
+            }
+            __syncthreads();
+        }
+    }
+    for (int i = threadIdx.x; i < k; i += kTrainThreads) {
+        const uint32_t c = (uint32_t)(keys[i] & 0xffffffffu);
+        idx_out[(size_t)e * k + i] = (int32_t)c;
+        lg_out[(size_t)e * k + i] = Le[c];
+    }
+}
+
+// Row statistics: stat[e] = {max_c L_{e,c}, sum_c exp(L_{e,c} - max)}.
+__global__ void __launch_bounds__(kTrainThreads) cov_rows_kernel(const float *__restrict__ L,
+                                                                  int C, float2 *__restrict__ stat) {
+    __shared__ float red[kTrainThreads / 32];
+    const int e = blockIdx.x;
+    const float *Le = L + (size_t)e * C;
+    float m = -INFINITY;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) m = fmaxf(m, Le[c]);
+    m = block_max_f(m, red);
+    float s = 0.f;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) s += expf(Le[c] - m);
+    s = block_sum_f(s, red);
+    if (threadIdx.x == 0) stat[e] = make_float2(m, s);
+}
+
+// Partial column sums: part[j][c] = sum over rows j kRowChunk .. + kRowChunk - 1
+// (in order) of p_{e,c}, in double; thread c of a 256-column block, chunk
+// j = blockIdx.y (coalesced row segments).
+__global__ void __launch_bounds__(256) cov_cols_kernel(const float *__restrict__ L, int R, int C,
+                                                       const float2 *__restrict__ stat,
+                                                       double *__restrict__ part) {
+    const int c = blockIdx.x * 256 + threadIdx.x;
+    if (c >= C) return;
+    const int e0 = blockIdx.y * kRowChunk, e1 = min(R, e0 + kRowChunk);
+    double s = 0.0;
+#pragma unroll 8
+    for (int e = e0; e < e1; ++e) {
+        const float2 st = stat[e];
+        s += (double)(expf(L[(size_t)e * C + c] - st.x) / st.y);
+    }
+    part[(size_t)blockIdx.y * C + c] = s;
+}
+
+// u_c = (1/R) sum_j part[j][c], the chunks in order; kept in the part
+// buffer's row 0 (thread c alone reads column c).
+__global__ void __launch_bounds__(256) cov_usage_kernel(double *__restrict__ part, int R, int C,
+                                                        int chunks) {
+    const int c = blockIdx.x * 256 + threadIdx.x;
+    if (c >= C) return;
+    double t = 0.0;
+#pragma unroll 8
+    for (int j = 0; j < chunks; ++j) t += part[(size_t)j * C + c];
+    part[c] = t / (double)R;
+}
+
+// The loss and g_c = dL_cov/du_c from u; one CTA, double.
+__global__ void __launch_bounds__(kTrainThreads) cov_loss_kernel(const double *__restrict__ u,
+                                                                  int C, double eps,
+                                                                  float *__restrict__ loss,
+                                                                  float *__restrict__ u_out,
+                                                                  float *__restrict__ g) {
+    __shared__ double red[kTrainThreads / 32];
+    double s = 0.0;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) s += u[c];
+    const double ubar = block_sum_d(s, red) / (double)C;
+    double S = 0.0, dev = 0.0;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) {
+        const double d = u[c] - ubar;
+        S += d * d;
+        dev += d;
+    }
+    S = block_sum_d(S, red);
+    dev = block_sum_d(dev, red);
+    const double D = ubar * ubar + eps;
+    if (threadIdx.x == 0) *loss = (float)(S / D);
+    // g_c = 2 (u_c - ubar) / D + shift, the shift (the same for every c) from
+    // the dependence of ubar on u; the divisions once per CTA
+    const double twoD = 2.0 / D;
+    const double shift = -2.0 * dev / ((double)C * D) - 2.0 * ubar * S / ((double)C * D * D);
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) {
+        if (u_out) u_out[c] = (float)u[c];
+        if (g) g[c] = (float)(twoD * (u[c] - ubar) + shift);
+    }
+}
+
+// dL_cov/dL_{e,c} = (1/R) p_{e,c} (g_c - sum_c' p_{e,c'} g_c'), one CTA per row.
+__global__ void __launch_bounds__(kTrainThreads) cov_grad_kernel(const float *__restrict__ L, int R,
+                                                                  int C,
+                                                                  const float2 *__restrict__ stat,
+                                                                  const float *__restrict__ g,
+                                                                  float *__restrict__ grad) {
+    __shared__ float red[kTrainThreads / 32];
+    const int e = blockIdx.x;
+    const float *Le = L + (size_t)e * C;
+    const float2 st = stat[e];
+    float dot = 0.f;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) dot += expf(Le[c] - st.x) / st.y * g[c];
+    dot = block_sum_f(dot, red);
+    const float inv_R = 1.f / (float)R;
+    for (int c = threadIdx.x; c < C; c += kTrainThreads) {
+        const float p = expf(Le[c] - st.x) / st.y;
+        grad[(size_t)e * C + c] = p * (g[c] - dot) * inv_R;
+    }
+}
+
+}  // namespace
+
+int topk_padded(int C) {
+    int cp = 1;
+    while (cp < C) cp <<= 1;
+    return cp;
+}
+
+// Workspace of the support-maintenance calls: the error word, the row
+// statistics, u in double and g.
+size_t train_ws_bytes(int R, int C) {
+    const size_t chunks = (size_t)(R + kRowChunk - 1) / kRowChunk;
+    return align_up(16, 256) + align_up((size_t)R * 8, 256) + align_up(chunks * C * 8, 256) +
+           align_up((size_t)C * 4, 256);
+}
+
+cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float *lg,
+                        uint32_t *err, cudaStream_t s) {
+    const int CP = topk_padded(C);
+    const size_t smem = (size_t)CP * 8;
+    cudaError_t e = cudaFuncSetAttribute(topk_rows_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    topk_rows_kernel<<<R, kTrainThreads, smem, s>>>(L, C, CP, k, idx, lg, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_coverage(const float *L, int R, int C, double eps, float *loss, float *u,
+                            float *grad, unsigned char *ws, cudaStream_t s) {
+    const int chunks = (R + kRowChunk - 1) / kRowChunk;
+    float2 *stat = reinterpret_cast<float2 *>(ws + align_up(16, 256));
+    double *ud = reinterpret_cast<double *>(ws + align_up(16, 256) + align_up((size_t)R * 8, 256));
+    float *g = reinterpret_cast<float *>(ws + align_up(16, 256) + align_up((size_t)R * 8, 256) +
+                                         align_up((size_t)chunks * C * 8, 256));
+    cov_rows_kernel<<<R, kTrainThreads, 0, s>>>(L, C, stat);
+    cov_cols_kernel<<<dim3((C + 255) / 256, chunks), 256, 0, s>>>(L, R, C, stat, ud);
+    cov_usage_kernel<<<(C + 255) / 256, 256, 0, s>>>(ud, R, C, chunks);
+    cov_loss_kernel<<<1, kTrainThreads, 0, s>>>(ud, C, eps, loss, u, grad ? g : nullptr);
+    if (grad) cov_grad_kernel<<<R, kTrainThreads, 0, s>>>(L, R, C, stat, g, grad);
+    return cudaGetLastError();
+}
+
+}  // namespace moce

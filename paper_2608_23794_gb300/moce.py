@@ -70,6 +70,9 @@ def library():
             "moce_forward_kernel": ([P, I, I, I, I, I, I, I, I], ctypes.c_char_p),
             "moce_forward_noalloc": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F, P, P], I),
             "moce_noalloc_check_device_error": ([P], I),
+            "moce_train_workspace_bytes": ([I, I], S),
+            "moce_topk_supports": ([P, I, I, I, P, P, P, S, P], I),
+            "moce_coverage_loss": ([P, I, I, F, P, P, P, P, S, P], I),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -289,6 +292,46 @@ def moce_forward_noalloc(x: torch.Tensor, layout: str, packed: PackedSupports, W
                                           float(tau_max), _ptr(y), _stream(stream)),
            "moce_forward_noalloc")
     return y
+
+
+def _train_ws(C_in: int, C_out: int, device) -> torch.Tensor:
+    nbytes = library().moce_train_workspace_bytes(C_in, C_out)
+    if nbytes == 0:
+        raise MoceError(MOCE_ERR_INVALID_VALUE, "moce_train_workspace_bytes")
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def moce_topk_supports(logits: torch.Tensor, k: int, stream=None):
+    """Eq. (support): the top-k channels of each row of logits [C_out, C_in], in deployment order.
+
+    Returns (packed_idx int32 [C_out, k], packed_logits float32 [C_out, k]). Synchronous.
+    """
+    logits = logits.contiguous()
+    if logits.dtype != torch.float32 or logits.dim() != 2:
+        raise ValueError("logits must be float32 [C_out, C_in]")
+    R, C = logits.shape
+    idx = torch.empty((R, k), dtype=torch.int32, device=logits.device)
+    lg = torch.empty((R, k), dtype=torch.float32, device=logits.device)
+    ws = _train_ws(C, R, logits.device)
+    _check(library().moce_topk_supports(_ptr(logits), C, R, k, _ptr(idx), _ptr(lg), _ptr(ws),
+                                        ws.numel(), _stream(stream)), "moce_topk_supports")
+    return idx, lg
+
+
+def moce_coverage_loss(logits: torch.Tensor, eps: float, grad: bool = True, stream=None):
+    """Sec. 3.4 coverage regularizer: (loss [1], usage u [C_in], dloss/dlogits [C_out, C_in] or None)."""
+    logits = logits.contiguous()
+    if logits.dtype != torch.float32 or logits.dim() != 2:
+        raise ValueError("logits must be float32 [C_out, C_in]")
+    R, C = logits.shape
+    loss = torch.empty(1, dtype=torch.float32, device=logits.device)
+    usage = torch.empty(C, dtype=torch.float32, device=logits.device)
+    g = torch.empty((R, C), dtype=torch.float32, device=logits.device) if grad else None
+    ws = _train_ws(C, R, logits.device)
+    _check(library().moce_coverage_loss(_ptr(logits), C, R, float(eps), _ptr(loss), _ptr(usage),
+                                        _ptr(g) if g is not None else None, _ptr(ws), ws.numel(),
+                                        _stream(stream)), "moce_coverage_loss")
+    return loss, usage, g
 
 
 def moce_noalloc_check_device_error(stream=None):
