@@ -66,8 +66,11 @@ def _load():
         lib.moce_oracle_bruteforce_forward.argtypes = [P, I, I, I, I, I, I, I, P, P, P, P, F, D, D,
                                                        P]
         lib.moce_oracle_coverage.argtypes = [I, I, P, D, P, P, P]
+        lib.moce_oracle_backward.argtypes = [P, P, I, I, I, I, I, I, I, P, P, P, I, P, P, P, F, D,
+                                             D, P, P, P, P, P, P]
         for fn in (lib.moce_oracle_topk, lib.moce_oracle_pack, lib.moce_oracle_forward,
-                   lib.moce_oracle_bruteforce_forward, lib.moce_oracle_coverage):
+                   lib.moce_oracle_bruteforce_forward, lib.moce_oracle_coverage,
+                   lib.moce_oracle_backward):
             fn.restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -113,6 +116,42 @@ def coverage(L: np.ndarray, eps: float, grad: bool = True):
     if st != OK:
         raise OracleError(st, "coverage")
     return float(loss[0]), u, g
+
+
+def backward(x: np.ndarray, dy: np.ndarray, layout: str, packed_idx, packed_logits, resid, W1,
+             b1, w2, b2: float, tau_min: float, tau_max: float):
+    """Gradients of the layer (static supports, Sec. 3.2) for the upstream gradient dy.
+
+    Returns a dict of float64 arrays: dx (the shape of x), dlogit [R, k], dW1 [k, k],
+    db1 [k], dw2 [k], db2 (float).
+    """
+    x = _c(x, np.float32)
+    dy = _c(dy, np.float32)
+    if layout == "nhwc":
+        N, H, W, C = x.shape
+    else:
+        N, C, H, W = x.shape
+    pidx = _c(packed_idx, np.int32)
+    R, k = pidx.shape
+    plog = _c(packed_logits, np.float32)
+    resid = _c(resid, np.int32)
+    W1 = _c(W1, np.float32)
+    b1 = _c(b1, np.float32)
+    w2 = _c(w2, np.float32)
+    dx = np.empty(x.shape, np.float64)
+    dlogit = np.empty((R, k), np.float64)
+    dW1 = np.empty((k, k), np.float64)
+    db1 = np.empty(k, np.float64)
+    dw2 = np.empty(k, np.float64)
+    db2 = np.zeros(1, np.float64)
+    st = _load().moce_oracle_backward(_p(x), _p(dy), N, H, W, C, _LAYOUT[layout], R, k, _p(pidx),
+                                      _p(plog), _p(resid) if resid.size else None, int(resid.size),
+                                      _p(W1), _p(b1), _p(w2), float(b2), float(tau_min),
+                                      float(tau_max), _p(dx), _p(dlogit), _p(dW1), _p(db1),
+                                      _p(dw2), _p(db2))
+    if st != OK:
+        raise OracleError(st, "backward")
+    return {"dx": dx, "dlogit": dlogit, "dW1": dW1, "db1": db1, "dw2": dw2, "db2": float(db2[0])}
 
 
 def pack(support_idx: np.ndarray, support_logits: np.ndarray, C: int):
@@ -261,7 +300,8 @@ class _use_library:
         # reuse the argtypes of the real build
         for name in ("moce_oracle_topk", "moce_oracle_pack", "moce_oracle_pool", "moce_oracle_gate",
                      "moce_oracle_weights", "moce_oracle_mix", "moce_oracle_forward",
-                     "moce_oracle_bruteforce_forward", "moce_oracle_coverage"):
+                     "moce_oracle_bruteforce_forward", "moce_oracle_coverage",
+                     "moce_oracle_backward"):
             src, dst = getattr(self._saved, name), getattr(lib, name)
             dst.argtypes, dst.restype = src.argtypes, src.restype
         _lib = lib

@@ -22,6 +22,10 @@
  *   residual  Eq. (res), Sec. 3.4           mean of X over U, 0 if U is empty
  *   coverage  Sec. 3.4                      L_cov over the full routing matrix and
  *             its gradient with respect to every logit (chain rule, written out)
+ *   backward  Sec. 3.2 (the task loss differentiates through the selected logit
+ *             values; no gradient through the indices): the gradients of a
+ *             scalar loss with respect to x, the selected logits and the gate
+ *             parameters, given dy, by the chain rule through the steps above
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - ties between equal logits order by ascending channel index; -0.0 and
@@ -31,7 +35,8 @@
  *   - the softmax subtracts the largest support logit before exponentiating,
  *     which leaves Eq. (weights) unchanged;
  *   - U is listed in ascending channel order;
- *   - the coverage loss's epsilon is an argument (the paper does not print it).
+ *   - the coverage loss's epsilon is an argument (the paper does not print it);
+ *   - the derivative of ReLU at exactly 0 is taken as 0.
  *
  * Inputs are the exact values the device sees (bf16 inputs are decoded to
  * float first); all arithmetic is in double.
@@ -480,5 +485,147 @@ int moce_oracle_coverage(int C, int R, const float *L, double eps, double *loss,
     free(p);
     free(u);
     free(g);
+    return ORACLE_OK;
+}
+
+/*
+ * Backward of the layer with static supports (Sec. 3.2: gradients reach the
+ * selected logit values, never the indices). Given dy = dJ/dy (the layout and
+ * shape of y) for a scalar J, returns by the chain rule through pool, gate,
+ * weights, routed mix and residual, per example n:
+ *   da_{e,i}  = sum_p dy_{p,e} x_{p,S_e[i]}                          Eq. (expert)
+ *   ds_{e,i}  = a_{e,i} (da_{e,i} - sum_j a_{e,j} da_{e,j}),  s = L / tau   Eq. (weights)
+ *   dL_{e,i} += ds_{e,i} / tau_e;  dtau_e = -sum_i ds_{e,i} L_{e,i} / tau_e^2
+ *   dg_e      = dtau_e (tau_max - tau_min) sigma_e (1 - sigma_e)       Eq. (tau)
+ *   dw2_j    += dg_e r_{e,j};  db2 += dg_e;  dh_{e,j} = dg_e w2_j [h_{e,j} > 0]
+ *   dW1_{j,i}+= dh_{e,j} u_{e,i};  db1_j += dh_{e,j};  du_{e,i} = sum_j W1_{j,i} dh_{e,j}
+ *   dz_c      = sum over (e, i) with S_e[i] = c of du_{e,i}            (u = z[S_e])
+ *   dx_{p,c}  = sum over (e, i) with S_e[i] = c of a_{e,i} dy_{p,e}
+ *               + [c in U] dy_{p,R} / |U| + dz_c / HW                 Eq. (res), GAP
+ * dx has the layout of x; dlogit [R][k] (packed order), dW1 [k][k] (row j =
+ * hidden unit j), db1 [k], dw2 [k], db2 [1] are sums over the batch.
+ */
+int moce_oracle_backward(const float *x, const float *dy, int N, int H, int W, int C, int layout,
+                         int R, int k, const int32_t *packed_idx, const float *packed_logits,
+                         const int32_t *resid, int n_resid, const float *W1, const float *b1,
+                         const float *w2, float b2, double tau_min, double tau_max, double *dx,
+                         double *dlogit, double *dW1, double *db1, double *dw2, double *db2)
+{
+    if (N < 0 || H < 0 || W < 0 || C < 1 || R < 1 || k < 1 || k > C || n_resid < 0 ||
+        n_resid > C || (layout != 0 && layout != 1) || !dx || !dlogit || !dW1 || !db1 || !dw2 ||
+        !db2)
+        return ORACLE_BAD_ARG;
+    const int HW = H * W, E = R + 1;
+    double *z = (double *)malloc(sizeof(double) * (size_t)C);
+    double *u = (double *)malloc(sizeof(double) * (size_t)k);
+    double *hpre = (double *)malloc(sizeof(double) * (size_t)k);
+    double *a = (double *)malloc(sizeof(double) * (size_t)k);
+    double *da = (double *)malloc(sizeof(double) * (size_t)k);
+    double *dh = (double *)malloc(sizeof(double) * (size_t)k);
+    double *dz = (double *)malloc(sizeof(double) * (size_t)C);
+    double *aall = (double *)malloc(sizeof(double) * ((size_t)R * k + 1));
+    if (!z || !u || !hpre || !a || !da || !dh || !dz || !aall) {
+        free(z); free(u); free(hpre); free(a); free(da); free(dh); free(dz); free(aall);
+        return ORACLE_NO_MEMORY;
+    }
+    for (int i = 0; i < R * k; ++i)
+        dlogit[i] = 0.0;
+    for (int i = 0; i < k * k; ++i)
+        dW1[i] = 0.0;
+    for (int j = 0; j < k; ++j) {
+        db1[j] = 0.0;
+        dw2[j] = 0.0;
+    }
+    *db2 = 0.0;
+    for (int n = 0; n < N; ++n) {
+        /* forward of example n: z, then per expert u, h, g, sigma, tau, a */
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int p = 0; p < HW; ++p)
+                s += (double)x[x_at(layout, n, p, c, HW, C)];
+            z[c] = s / (double)HW;
+            dz[c] = 0.0;
+        }
+        for (int e = 0; e < R; ++e) {
+            const int32_t *S = packed_idx + (size_t)e * k;
+            const float *L = packed_logits + (size_t)e * k;
+            for (int i = 0; i < k; ++i)
+                u[i] = z[S[i]];
+            double g = (double)b2;
+            for (int j = 0; j < k; ++j) {
+                double t = (double)b1[j];
+                for (int i = 0; i < k; ++i)
+                    t += (double)W1[(size_t)j * k + i] * u[i];
+                hpre[j] = t;
+                g += (double)w2[j] * (t > 0.0 ? t : 0.0);
+            }
+            const double sig = 1.0 / (1.0 + exp(-g));
+            const double tau = tau_min + (tau_max - tau_min) * sig;
+            double m = (double)L[0];
+            for (int i = 1; i < k; ++i)
+                if ((double)L[i] > m)
+                    m = (double)L[i];
+            double sum = 0.0;
+            for (int i = 0; i < k; ++i) {
+                a[i] = exp(((double)L[i] - m) / tau);
+                sum += a[i];
+            }
+            for (int i = 0; i < k; ++i) {
+                a[i] /= sum;
+                aall[(size_t)e * k + i] = a[i];
+            }
+            /* backward: routed mix -> weights -> temperature -> gate */
+            for (int i = 0; i < k; ++i) {
+                double s = 0.0;
+                for (int p = 0; p < HW; ++p)
+                    s += (double)dy[x_at(layout, n, p, e, HW, E)] *
+                         (double)x[x_at(layout, n, p, S[i], HW, C)];
+                da[i] = s;
+            }
+            double ada = 0.0;
+            for (int i = 0; i < k; ++i)
+                ada += a[i] * da[i];
+            double dtau = 0.0;
+            for (int i = 0; i < k; ++i) {
+                const double ds = a[i] * (da[i] - ada);
+                dlogit[(size_t)e * k + i] += ds / tau;
+                dtau -= ds * (double)L[i] / (tau * tau);
+            }
+            const double dg = dtau * (tau_max - tau_min) * sig * (1.0 - sig);
+            *db2 += dg;
+            for (int j = 0; j < k; ++j) {
+                const double r = hpre[j] > 0.0 ? hpre[j] : 0.0;
+                dw2[j] += dg * r;
+                dh[j] = hpre[j] > 0.0 ? dg * (double)w2[j] : 0.0;
+                db1[j] += dh[j];
+                for (int i = 0; i < k; ++i)
+                    dW1[(size_t)j * k + i] += dh[j] * u[i];
+            }
+            for (int i = 0; i < k; ++i) {
+                double du = 0.0;
+                for (int j = 0; j < k; ++j)
+                    du += (double)W1[(size_t)j * k + i] * dh[j];
+                dz[S[i]] += du;
+            }
+        }
+        /* dx: the routed experts' weights, the residual mean and the pool */
+        for (int p = 0; p < HW; ++p)
+            for (int c = 0; c < C; ++c)
+                dx[x_at(layout, n, p, c, HW, C)] = dz[c] / (double)HW;
+        for (int p = 0; p < HW; ++p) {
+            for (int e = 0; e < R; ++e) {
+                const double d = (double)dy[x_at(layout, n, p, e, HW, E)];
+                for (int i = 0; i < k; ++i)
+                    dx[x_at(layout, n, p, packed_idx[(size_t)e * k + i], HW, C)] +=
+                        aall[(size_t)e * k + i] * d;
+            }
+            if (n_resid > 0) {
+                const double d = (double)dy[x_at(layout, n, p, R, HW, E)] / (double)n_resid;
+                for (int j = 0; j < n_resid; ++j)
+                    dx[x_at(layout, n, p, resid[j], HW, C)] += d;
+            }
+        }
+    }
+    free(z); free(u); free(hpre); free(a); free(da); free(dh); free(dz); free(aall);
     return ORACLE_OK;
 }

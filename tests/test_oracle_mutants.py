@@ -24,7 +24,8 @@ MUTANTS = {
     "gate_relu_dropped": ("h[j] = s > 0.0 ? s : 0.0;", "h[j] = s;"),
     "gate_b2_dropped": ("double g = (double)b2;\n            for (int j = 0; j < k; ++j)\n                g += (double)w2[j] * h[j];",
                         "double g = 0.0;\n            for (int j = 0; j < k; ++j)\n                g += (double)w2[j] * h[j];"),
-    "sigmoid_sign": ("double sig = 1.0 / (1.0 + exp(-g));", "double sig = 1.0 / (1.0 + exp(g));"),
+    "sigmoid_sign": ("double sig = 1.0 / (1.0 + exp(-g));\n            if (g_out)",
+                     "double sig = 1.0 / (1.0 + exp(g));\n            if (g_out)"),
     "tau_reversed": ("tau[(size_t)n * R + e] = tau_min + (tau_max - tau_min) * sig;",
                      "tau[(size_t)n * R + e] = tau_max - (tau_max - tau_min) * sig;"),
     "pool_not_divided": ("z[(size_t)n * C + c] = s / (double)HW;", "z[(size_t)n * C + c] = s;"),
@@ -47,6 +48,18 @@ MUTANTS = {
     # softmax Jacobian, so dropping one is not a mistake; flipping the
     # per-channel deviation is)
     "coverage_grad_deviation_sign": ("g[c] = 2.0 * (u[c] - ubar) / D", "g[c] = 2.0 * (ubar - u[c]) / D"),
+    "backward_softmax_mean_dropped": ("const double ds = a[i] * (da[i] - ada);",
+                                      "const double ds = a[i] * da[i];"),
+    "backward_dtau_sign": ("dtau -= ds * (double)L[i] / (tau * tau);",
+                           "dtau += ds * (double)L[i] / (tau * tau);"),
+    "backward_pool_not_divided": ("dx[x_at(layout, n, p, c, HW, C)] = dz[c] / (double)HW;",
+                                  "dx[x_at(layout, n, p, c, HW, C)] = dz[c];"),
+    "backward_relu_mask_dropped": ("dh[j] = hpre[j] > 0.0 ? dg * (double)w2[j] : 0.0;",
+                                   "dh[j] = dg * (double)w2[j];"),
+    "backward_du_uses_W1_rows": ("du += (double)W1[(size_t)j * k + i] * dh[j];",
+                                 "du += (double)W1[(size_t)i * k + j] * dh[j];"),
+    "backward_residual_not_divided": ("const double d = (double)dy[x_at(layout, n, p, R, HW, E)] / (double)n_resid;",
+                                      "const double d = (double)dy[x_at(layout, n, p, R, HW, E)];"),
     "coverage_grad_softmax_jacobian_dot_dropped": ("p[(size_t)e * C + c] * (g[c] - dot) / (double)R;",
                                                    "p[(size_t)e * C + c] * g[c] / (double)R;"),
 }
@@ -73,6 +86,8 @@ PIN_CHECKS = [
     lambda: pins.test_coverage_one_expert_two_channels_closed_form(2.5, -1.0),
     pins.test_coverage_row_shift_and_channel_permutation,
     pins.test_coverage_equals_numpy_definition_and_finite_differences,
+    lambda: pins.test_backward_equals_central_differences("nhwc"),
+    pins.test_backward_constant_temperature_is_the_transposed_linear_map,
 ]
 
 

@@ -385,3 +385,97 @@ def test_layouts_agree():
     y_nchw = oracle.forward(lay.x, "nchw", *args)
     y_nhwc = oracle.forward(synth.x_to_layout(lay.x, "nchw", "nhwc"), "nhwc", *args)
     assert np.array_equal(synth.x_to_layout(y_nhwc, "nhwc", "nchw"), y_nchw)
+
+
+# ---------------------------------------------------------------- backward (Sec. 3.2)
+
+
+def _bwd_layer(layout, seed=0, N=2, H=3, W=4, C=12, R=5, k=3):
+    rng = np.random.default_rng(seed)
+    shape = (N, H, W, C) if layout == "nhwc" else (N, C, H, W)
+    x = rng.standard_normal(shape).astype(np.float32)
+    idx = np.stack([rng.permutation(C - 2)[:k] for _ in range(R)]).astype(np.int32)  # |U| >= 2
+    lg = rng.standard_normal((R, k)).astype(np.float32)
+    pidx, plog, resid = oracle.pack(idx, lg, C)
+    W1 = (rng.standard_normal((k, k)) / np.sqrt(k)).astype(np.float32)
+    b1 = (0.3 * rng.standard_normal(k)).astype(np.float32)
+    w2 = rng.standard_normal(k).astype(np.float32)
+    b2 = np.float32(0.2)
+    yshape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+    dy = rng.standard_normal(yshape).astype(np.float32)
+    return x, pidx, plog, resid, W1, b1, w2, b2, dy
+
+
+def _J(layout, x, pidx, plog, resid, W1, b1, w2, b2, dy, tmin=0.2, tmax=6.0):
+    y = oracle.forward(x, layout, pidx, plog, resid, W1, b1, w2, float(b2), tmin, tmax)
+    return float((y * dy.astype(np.float64)).sum())
+
+
+@pytest.mark.parametrize("layout", ["nhwc", "nchw"])
+def test_backward_equals_central_differences(layout):
+    x, pidx, plog, resid, W1, b1, w2, b2, dy = _bwd_layer(layout, seed=3)
+    g = oracle.backward(x, dy, layout, pidx, plog, resid, W1, b1, w2, float(b2), 0.2, 6.0)
+    args = dict(x=x, pidx=pidx, plog=plog, resid=resid, W1=W1, b1=b1, w2=w2, b2=np.array([b2]),
+                dy=dy)
+    h = 2.0 ** -12  # exact in float32 for these magnitudes
+
+    def fd(name, flat_i):
+        a = {kk: (v.copy() if isinstance(v, np.ndarray) else v) for kk, v in args.items()}
+        arr = a[name].reshape(-1)
+        v0 = float(arr[flat_i])
+        arr[flat_i] = np.float32(v0 + h)
+        dp = float(arr[flat_i]) - v0
+        jp = _J(layout, a["x"], a["pidx"], a["plog"], a["resid"], a["W1"], a["b1"], a["w2"],
+                a["b2"][0], a["dy"])
+        arr[flat_i] = np.float32(v0 - h)
+        dm = v0 - float(arr[flat_i])
+        jm = _J(layout, a["x"], a["pidx"], a["plog"], a["resid"], a["W1"], a["b1"], a["w2"],
+                a["b2"][0], a["dy"])
+        return (jp - jm) / (dp + dm)
+
+    for name, got in [("x", g["dx"]), ("plog", g["dlogit"]), ("W1", g["dW1"]), ("b1", g["db1"]),
+                      ("w2", g["dw2"]), ("b2", np.array([g["db2"]]))]:
+        flat = got.reshape(-1)
+        want = np.array([fd(name, i) for i in range(flat.size)])
+        np.testing.assert_allclose(flat, want, rtol=1e-5, atol=1e-7, err_msg=name)
+
+
+def test_backward_constant_temperature_is_the_transposed_linear_map():
+    # tau_min = tau_max: tau does not depend on x or the gate, so the gate
+    # gradients vanish, dx = W_eff^T dy with W_eff the per-example dense map of
+    # Eq. (expert) and Eq. (res), and dlogit follows softmax(L / T) alone
+    x, pidx, plog, resid, W1, b1, w2, b2, dy = _bwd_layer("nhwc", seed=5)
+    T = 0.7
+    g = oracle.backward(x, dy, "nhwc", pidx, plog, resid, W1, b1, w2, float(b2), T, T)
+    for name in ("dW1", "db1", "dw2"):
+        assert np.all(g[name] == 0.0), name
+    assert g["db2"] == 0.0
+    R, k = pidx.shape
+    C = x.shape[-1]
+    A = sp_softmax(plog.astype(np.float64) / T, axis=1)
+    Weff = np.zeros((R + 1, C))
+    for e in range(R):
+        for i in range(k):
+            Weff[e, pidx[e, i]] += A[e, i]
+    if len(resid):
+        Weff[R, resid] = 1.0 / len(resid)
+    np.testing.assert_allclose(g["dx"], np.einsum("nhwe,ec->nhwc", dy.astype(np.float64), Weff),
+                               rtol=1e-12, atol=1e-12)
+    # dJ/dL_{e,i} = (1/T) a_i (da_i - sum_j a_j da_j), da_{e,i} = sum dy_e x_{S_e[i]}
+    da = np.einsum("nhwe,nhwei->ei", dy.astype(np.float64)[..., :R],
+                   x.astype(np.float64)[..., pidx])
+    want = A * (da - (A * da).sum(1, keepdims=True)) / T
+    np.testing.assert_allclose(g["dlogit"], want, rtol=1e-10, atol=1e-12)
+
+
+def test_backward_is_linear_in_dy():
+    x, pidx, plog, resid, W1, b1, w2, b2, dy = _bwd_layer("nhwc", seed=9)
+    dy2 = np.random.default_rng(1).standard_normal(dy.shape).astype(np.float32)
+    g1 = oracle.backward(x, dy, "nhwc", pidx, plog, resid, W1, b1, w2, float(b2), 0.2, 6.0)
+    g2 = oracle.backward(x, dy2, "nhwc", pidx, plog, resid, W1, b1, w2, float(b2), 0.2, 6.0)
+    g3 = oracle.backward(x, (dy + dy2).astype(np.float32), "nhwc", pidx, plog, resid, W1, b1, w2,
+                         float(b2), 0.2, 6.0)
+    # (dy + dy2 is rounded to float32: agreement to that rounding, relative to each array's scale)
+    for name in ("dx", "dlogit", "dW1", "db1", "dw2"):
+        want = g1[name] + g2[name]
+        np.testing.assert_allclose(g3[name], want, rtol=0, atol=1e-6 * np.abs(want).max())
