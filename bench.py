@@ -54,8 +54,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto",
                     help="kernel path of the forward (auto, stream, steps)")
-    ap.add_argument("--op", choices=["forward", "train"], default="forward",
-                    help="forward: the layer forward (the benchmark); train: TopK over the full "
+    ap.add_argument("--op", choices=["forward", "backward", "train"], default="forward",
+                    help="forward: the layer forward (the benchmark); backward: the layer's "
+                         "gradients for an upstream gradient; train: TopK over the full "
                          "routing matrix and the coverage loss with its gradient")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline leg")
@@ -606,12 +607,108 @@ def run_train(args, cfg):
     print(json.dumps(line), flush=True)
 
 
+def run_backward(args, cfg):
+    """The layer's backward with static supports (Sec. 3.2) at the workload's full size: device
+    time per call (inputs rotated so every call reads x and dy from HBM), GB/s of the algorithmic
+    bytes (x and dy read once, dx written once in fp32) against the HBM peak, and the oracle's
+    backward on one host core over a sample of examples."""
+    import numpy as np
+    import torch
+
+    from paper_2608_23794_gb300 import build as moce_build
+    from paper_2608_23794_gb300 import moce, synth
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    moce_build.build()
+    lay = synth.make_layer(cfg, seed=SEED)
+    dyv, dyb = synth.make_dy(cfg, seed=SEED)
+    s = 2 if cfg.dtype == "bf16" else 4
+    if cfg.dtype == "bf16":
+        x = torch.from_numpy(lay.x_bits.view(np.int16)).view(torch.bfloat16)
+        dy = torch.from_numpy(dyb.view(np.int16)).view(torch.bfloat16)
+    else:
+        x, dy = torch.from_numpy(lay.x), torch.from_numpy(dyv)
+    cu = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).to(device=dev, dtype=dt)
+    W1, b1, w2, b2 = (cu(lay.W1, torch.float32), cu(lay.b1, torch.float32),
+                      cu(lay.w2, torch.float32), cu(lay.b2, torch.float32))
+    packed = moce.moce_pack_supports(cu(lay.support_idx, torch.int32),
+                                     cu(lay.support_logits, torch.float32), cfg.C_in)
+    R, k, C = cfg.C_out, cfg.k, cfg.C_in
+    M = cfg.N * cfg.H * cfg.W
+    alg_bytes = M * C * s + M * (R + 1) * s + M * C * 4
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 132 * 2**20
+    n_rot = max(2, int(np.ceil(3 * l2 / alg_bytes)) + 1)
+    xs = [x.to(dev) for _ in range(n_rot)]
+    dys = [dy.to(dev) for _ in range(n_rot)]
+    f32 = dict(dtype=torch.float32, device=dev)
+    outs = [moce.Gradients(torch.empty(x.shape, **f32), torch.empty((R, k), **f32),
+                           torch.empty((k, k), **f32), torch.empty(k, **f32),
+                           torch.empty(k, **f32), torch.empty(1, **f32)) for _ in range(n_rot)]
+    ws = torch.empty(moce.moce_backward_workspace_bytes(cfg.N, cfg.H, cfg.W, C, R, k),
+                     dtype=torch.uint8, device=dev)
+    bwd = lambda i: moce.moce_backward(xs[i % n_rot], dys[i % n_rot], cfg.layout, packed, W1, b1,
+                                       w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
+                                       out=outs[i % n_rot])
+    for i in range(max(3, args.warmup)):
+        bwd(i)
+    torch.cuda.synchronize()
+    K = max(3, min(args.steps, 500))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(gpu_uuid(torch, dev))
+    sampler.start()
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    e0.record()
+    for i in range(K):
+        bwd(i)
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    us = e0.elapsed_time(e1) * 1e3 / K
+    peaks, _ = measured_peaks()
+    gbs = alg_bytes / us / 1e3
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        pidx, plog, resid = oracle.pack(lay.support_idx, lay.support_logits, C)
+        n_ex, spent = 0, 0.0
+        while n_ex < cfg.N and spent < min(args.cpu_seconds, 20.0):
+            t0 = time.perf_counter()
+            oracle.backward(lay.x[n_ex:n_ex + 1], dyv[n_ex:n_ex + 1], cfg.layout, pidx, plog,
+                            resid, lay.W1, lay.b1, lay.w2, float(lay.b2[0]), cfg.tau_min,
+                            cfg.tau_max)
+            spent += time.perf_counter() - t0
+            n_ex += 1
+        cpu = {"value": spent / n_ex * cfg.N * 1e6, "unit": "µs per backward (extrapolated)",
+               "cores": 1, "kind": "oracle",
+               "sample": f"{n_ex} of {cfg.N} examples, one core, scaled to the whole batch"}
+    line = {"metric": "MoCE backward µs/layer (static supports) & GB/s of algorithmic bytes",
+            "value": gbs, "unit": UNIT, "n_gpus": 1, "steps": K, "warmup": args.warmup,
+            "ms_per_step": us / 1e3, "us_per_layer": us, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": DATA[cfg.activation],
+            "config": {"workload": cfg.name, "N": cfg.N, "H": cfg.H, "W": cfg.W, "C_in": C,
+                       "C_out": R, "k": k, "storage_dtype": cfg.dtype, "layout": cfg.layout,
+                       "op": "backward", "l2": f"{n_rot} rotating input copies (> L2)"},
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "traffic": None,
+                         "note": "whole backward call (all its kernels), algorithmic bytes "
+                                 "x + dy + dx(fp32)"},
+            "clocks": clocks, "gpu_launches": None, "cpu_baseline": cpu}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     from paper_2608_23794_gb300 import synth
     cfg = synth.CONFIGS[args.workload]
     if args.op == "train":
         run_train(args, cfg)
+        return
+    if args.op == "backward":
+        run_backward(args, cfg)
         return
     if args.impl == "ours" and (cfg.dtype, cfg.layout) != ("bf16", "nhwc"):
         raise SystemExit(f"bench.py times bf16 NHWC layers; {cfg.name} is {cfg.dtype} {cfg.layout}")

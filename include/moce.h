@@ -1,5 +1,6 @@
 /*
- * moce.h - C ABI of the MoCE layer forward on NVIDIA GB300 (sm_103a).
+ * moce.h - C ABI of the MoCE layer (forward, backward, support maintenance)
+ * on NVIDIA GB300 (sm_103a).
  *
  * A Mixture of Channel Experts layer ("Mixture of Channel Experts: Static
  * Sparse Supports with Input-Adaptive Mixing for Pointwise Projections",
@@ -313,6 +314,42 @@ moce_status_t moce_topk_supports(const float *logits, int C_in, int C_out, int k
 moce_status_t moce_coverage_loss(const float *logits, int C_in, int C_out, float eps,
                                  float *loss, float *usage, float *grad, void *ws,
                                  size_t ws_bytes, moce_stream_t stream);
+
+/*
+ * Backward of the layer with static supports (Sec. 3.2: the loss reaches the
+ * selected logit values through the weights; the indices get no gradient).
+ * Given dy = dJ/dy of a scalar J, by the chain rule through the pool
+ * (Sec. 3.3), the gate and Eq. (tau), Eq. (weights), Eq. (expert) and Eq. (res):
+ *   da[n,e,i]  = sum_p dy[n,p,e] x[n,p,S_e[i]]
+ *   ds[n,e,i]  = a[n,e,i] (da[n,e,i] - sum_j a[n,e,j] da[n,e,j])
+ *   dlogits[e,i] = sum_n ds[n,e,i] / tau[n,e]
+ *   dtau[n,e]  = -sum_i ds[n,e,i] L[e,i] / tau[n,e]^2, and on through sigma,
+ *                w2, ReLU, W1, b1 to dW1, db1, dw2, db2 (summed over n, e)
+ *                and to the pooled descriptors z (du = W1^T dh)
+ *   dx[n,p,c]  = sum_{(e,i): S_e[i]=c} a[n,e,i] dy[n,p,e]
+ *                + [c in U] dy[n,p,C_out] / |U| + dz[n,c] / (H W)
+ * Arguments as moce_forward (x, supports, U, gate parameters, tau range), plus
+ *   dy      device, dtype and layout of y (C_out + 1 channels)
+ *   dx      device fp32 [N][H][W][C_in] (NHWC) or [N][C_in][H][W] (NCHW) out
+ *   dlogits device fp32 [C_out][k] out, in packed order
+ *   dW1     device fp32 [k][k] out (row j = hidden unit j), db1 / dw2 [k] out,
+ *   db2     device fp32 [1] out
+ * Every output is overwritten (not accumulated). With N = 0 or H W = 0 the
+ * parameter gradients are zero. Every sum runs in a fixed order: two calls
+ * give the same bits. ws: moce_backward_workspace_bytes, 256-byte aligned,
+ * no initialisation needed. C_in + C_out <= 5688 and C_out <= 3400
+ * (MOCE_ERR_UNSUPPORTED beyond: tiles staged in shared memory; the
+ * workspace size is then 0). Asynchronous.
+ */
+size_t moce_backward_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k);
+moce_status_t moce_backward(const void *x, const void *dy, int N, int H, int W, int C_in,
+                            int C_out, int k, moce_dtype_t dtype, moce_layout_t layout,
+                            const int32_t *packed_idx, const float *packed_logits,
+                            const int32_t *resid_idx, int n_resid, const float *W1,
+                            const float *b1, const float *w2, const float *b2, float tau_min,
+                            float tau_max, float *dx, float *dlogits, float *dW1, float *db1,
+                            float *dw2, float *db2, void *ws, size_t ws_bytes,
+                            moce_stream_t stream);
 
 /*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word the

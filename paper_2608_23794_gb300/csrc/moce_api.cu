@@ -276,6 +276,47 @@ moce_status_t moce_coverage_loss(const float *logits, int C_in, int C_out, float
                                        reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t moce_backward_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k) {
+    if (!shape_ok(N, H, W, C_in, C_out, k)) return 0;
+    return backward_ws_bytes(N, H * W, C_in, C_out, k);
+}
+
+moce_status_t moce_backward(const void *x, const void *dy, int N, int H, int W, int C_in,
+                            int C_out, int k, moce_dtype_t dtype, moce_layout_t layout,
+                            const int32_t *packed_idx, const float *packed_logits,
+                            const int32_t *resid_idx, int n_resid, const float *W1,
+                            const float *b1, const float *w2, const float *b2, float tau_min,
+                            float tau_max, float *dx, float *dlogits, float *dW1, float *db1,
+                            float *dw2, float *db2, void *ws, size_t ws_bytes,
+                            moce_stream_t stream) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
+        !tau_ok(tau_min, tau_max))
+        return MOCE_ERR_INVALID_VALUE;
+    if (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
+    if (!dlogits || !dW1 || !db1 || !dw2 || !db2) return MOCE_ERR_INVALID_VALUE;
+    const size_t need = backward_ws_bytes(N, H * W, C_in, C_out, k);
+    if (need == 0) return MOCE_ERR_UNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int HW = H * W;
+    if (N == 0 || HW == 0) {
+        cudaError_t err = cudaMemsetAsync(dlogits, 0, (size_t)C_out * k * 4, s);
+        if (err == cudaSuccess) err = cudaMemsetAsync(dW1, 0, (size_t)k * k * 4, s);
+        if (err == cudaSuccess) err = cudaMemsetAsync(db1, 0, (size_t)k * 4, s);
+        if (err == cudaSuccess) err = cudaMemsetAsync(dw2, 0, (size_t)k * 4, s);
+        if (err == cudaSuccess) err = cudaMemsetAsync(db2, 0, 4, s);
+        return cuda_status(err);
+    }
+    if (!x || !dy || !dx || !packed_idx || !packed_logits || !W1 || !b1 || !w2 || !b2 || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    if (ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u)) return MOCE_ERR_INVALID_VALUE;
+    const cudaError_t err = launch_backward(
+        x, dy, N, HW, C_in, C_out, k, dtype, layout, packed_idx, packed_logits, resid_idx, n_resid,
+        W1, b1, w2, b2, tau_min, tau_max, dx, dlogits, dW1, db1, dw2, db2,
+        static_cast<unsigned char *>(ws), s);
+    if (err == cudaErrorNotSupported) return MOCE_ERR_UNSUPPORTED;
+    return cuda_status(err);
+}
+
 moce_status_t moce_check_device_error(const void *ws, size_t ws_bytes, moce_stream_t stream) {
     if (!ws || ws_bytes < kCtrlWords * 4) return MOCE_ERR_INVALID_VALUE;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

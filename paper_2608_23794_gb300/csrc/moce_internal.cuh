@@ -147,6 +147,16 @@ cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float
 cudaError_t launch_coverage(const float *L, int R, int C, double eps, float *loss, float *u,
                             float *grad, unsigned char *ws, cudaStream_t s);
 
+// Backward with static supports (moce_backward.cu); 0 / cudaErrorNotSupported
+// when a staged tile does not fit.
+size_t backward_ws_bytes(int N, int HW, int C, int R, int k);
+cudaError_t launch_backward(const void *x, const void *dy, int N, int HW, int C, int R, int k,
+                            moce_dtype_t dt, moce_layout_t lay, const int32_t *pidx,
+                            const float *plog, const int32_t *resid, int nU, const float *W1,
+                            const float *b1, const float *w2, const float *b2, float tmin,
+                            float tmax, float *dx, float *dlogit, float *dW1, float *db1,
+                            float *dw2, float *db2, unsigned char *ws, cudaStream_t s);
+
 cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
                           const int32_t *pidx, const float *plog, const int32_t *resid, int nU,
                           const float *W1, const float *b1, const float *w2, const float *b2,

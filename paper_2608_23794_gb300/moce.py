@@ -73,6 +73,9 @@ def library():
             "moce_train_workspace_bytes": ([I, I], S),
             "moce_topk_supports": ([P, I, I, I, P, P, P, S, P], I),
             "moce_coverage_loss": ([P, I, I, F, P, P, P, P, S, P], I),
+            "moce_backward_workspace_bytes": ([I, I, I, I, I, I], S),
+            "moce_backward": ([P, P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F,
+                               P, P, P, P, P, P, P, S, P], I),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -332,6 +335,54 @@ def moce_coverage_loss(logits: torch.Tensor, eps: float, grad: bool = True, stre
                                         _ptr(g) if g is not None else None, _ptr(ws), ws.numel(),
                                         _stream(stream)), "moce_coverage_loss")
     return loss, usage, g
+
+
+@dataclass
+class Gradients:
+    dx: torch.Tensor        # float32, the shape and layout of x
+    dlogits: torch.Tensor   # float32 [C_out, k], packed order
+    dW1: torch.Tensor       # float32 [k, k]
+    db1: torch.Tensor       # float32 [k]
+    dw2: torch.Tensor       # float32 [k]
+    db2: torch.Tensor       # float32 [1]
+
+
+def moce_backward_workspace_bytes(N: int, H: int, W: int, C_in: int, C_out: int, k: int) -> int:
+    return int(library().moce_backward_workspace_bytes(N, H, W, C_in, C_out, k))
+
+
+def moce_backward(x: torch.Tensor, dy: torch.Tensor, layout: str, packed: PackedSupports, W1, b1,
+                  w2, b2, tau_min: float, tau_max: float, ws: torch.Tensor | None = None,
+                  out: Gradients | None = None, stream=None) -> Gradients:
+    """Gradients of the layer with static supports for the upstream gradient dy (Sec. 3.2).
+
+    ``out`` (optional) receives the gradients in place; every field is overwritten."""
+    N, H, W, C = _dims(x, layout)
+    R, k = packed.C_out, packed.k
+    if C != packed.C_in:
+        raise ValueError("x channels do not match the packed supports")
+    if dy.dtype != x.dtype or tuple(_dims(dy, layout)) != (N, H, W, R + 1):
+        raise ValueError("dy must have the dtype of x and the shape of y")
+    dev = x.device
+    f32 = dict(dtype=torch.float32, device=dev)
+    g = out or Gradients(torch.empty(x.shape, **f32), torch.empty((R, k), **f32),
+                         torch.empty((k, k), **f32), torch.empty(k, **f32), torch.empty(k, **f32),
+                         torch.empty(1, **f32))
+    if tuple(g.dx.shape) != tuple(x.shape) or g.dlogits.shape != (R, k) or g.dW1.shape != (k, k):
+        raise ValueError("gradient buffers do not match the layer")
+    if ws is None:
+        nbytes = moce_backward_workspace_bytes(N, H, W, C, R, k)
+        if nbytes == 0:
+            raise MoceError(MOCE_ERR_UNSUPPORTED, "moce_backward_workspace_bytes")
+        ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    _check(library().moce_backward(_ptr(x), _ptr(dy), N, H, W, C, R, k, _dtype(x),
+                                   _LAYOUTS[layout], _ptr(packed.packed_idx),
+                                   _ptr(packed.packed_logits), _ptr(packed.resid_idx),
+                                   packed.n_resid, _ptr(W1), _ptr(b1), _ptr(w2), _ptr(b2),
+                                   float(tau_min), float(tau_max), _ptr(g.dx), _ptr(g.dlogits),
+                                   _ptr(g.dW1), _ptr(g.db1), _ptr(g.dw2), _ptr(g.db2), _ptr(ws),
+                                   ws.numel(), _stream(stream)), "moce_backward")
+    return g
 
 
 def moce_noalloc_check_device_error(stream=None):

@@ -193,6 +193,21 @@ def make_layer(cfg: LayerConfig, seed: int = 0) -> SyntheticLayer:
     return SyntheticLayer(cfg, x, bits, sidx, slog, W1, b1, w2, b2)
 
 
+def make_dy(cfg: LayerConfig, seed: int = 0):
+    """Upstream gradient dJ/dy of a scalar J, the shape, layout and dtype of y
+    (C_out + 1 channels); returns (float32 values, bf16 bits or None)."""
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0x5EED]))
+    shape = (cfg.N, cfg.H, cfg.W, cfg.C_out + 1)
+    if cfg.layout == "nchw":
+        shape = (cfg.N, cfg.C_out + 1, cfg.H, cfg.W)
+    a = rng.standard_normal(shape, dtype=np.float32)
+    bits = None
+    if cfg.dtype == "bf16":
+        bits = bf16_bits(a)
+        a = bf16_to_f32(bits)
+    return a, bits
+
+
 def x_to_layout(x: np.ndarray, src: str, dst: str) -> np.ndarray:
     if src == dst:
         return x

@@ -127,6 +127,43 @@ def test_forward_path_selection_on_host(lib):
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3   # NCHW: pool, gate, mix
 
 
+def test_backward_rejects_bad_arguments_on_host(lib):
+    P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    wb = lib.moce_backward_workspace_bytes
+    wb.argtypes, wb.restype = [I] * 6, S
+    f = lib.moce_backward
+    f.argtypes = [P, P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F,
+                  P, P, P, P, P, P, P, S, P]
+    f.restype = I
+    assert wb(2, 4, 4, 64, 8, 4) > 0
+    assert wb(2, 4, 4, 64, 8, 0) == 0            # k < 1
+    assert wb(2, 4, 4, 6000, 8, 4) == 0          # staged da tile does not fit
+    assert wb(2, 4, 4, 64, 3500, 4) == 0         # staged dy tile of dx does not fit
+    fake = ctypes.c_void_p(0x1000)
+    good = dict(N=2, H=4, W=4, C=64, R=8, k=4, dt=1, lay=0, tmin=0.2, tmax=6.0, nU=3, dx=fake,
+                dW1=fake, ws=fake, wsb=1 << 40)
+
+    def call(**kw):
+        a = {**good, **kw}
+        return f(fake, fake, a["N"], a["H"], a["W"], a["C"], a["R"], a["k"], a["dt"], a["lay"],
+                 fake, fake, fake, a["nU"], fake, fake, fake, fake, a["tmin"], a["tmax"], a["dx"],
+                 fake, a["dW1"], fake, fake, fake, a["ws"], a["wsb"], None)
+
+    assert call(k=0) == 1
+    assert call(k=65) == 1
+    assert call(dt=5) == 1
+    assert call(lay=2) == 1
+    assert call(tmin=-1.0) == 1
+    assert call(nU=-1) == 1
+    assert call(nU=65) == 1
+    assert call(dW1=None) == 1
+    assert call(dx=None) == 1
+    assert call(ws=None) == 1
+    assert call(wsb=16) == 1                      # workspace too small
+    assert call(ws=ctypes.c_void_p(0x1010)) == 1  # not 256-byte aligned
+    assert call(C=6000, nU=0) == 3                # valid, no kernel for it
+
+
 def test_pack_rejects_bad_arguments_on_host(lib):
     f = lib.moce_pack_supports
     P, I = ctypes.c_void_p, ctypes.c_int
