@@ -36,6 +36,11 @@ CASES = {
     "tiny_f32_nchw": CFG["tiny_f32_nchw"],
     "ragged_f32_nhwc": LC("ragged_f32_nhwc", 3, 9, 11, 72, 9, 5, "f32", "nhwc", "relu", 60),
     "ragged_bf16_nchw": LC("ragged_bf16_nchw", 2, 13, 7, 48, 20, 40, "bf16", "nchw", "gelu", 48),
+    # NHWC bf16 tiles: a ragged last tile, and C % 8 != 0 (no 16-byte channel groups)
+    "ragged_bf16_nhwc": LC("ragged_bf16_nhwc", 3, 9, 11, 72, 9, 5, "bf16", "nhwc", "relu", 60),
+    "odd_c_bf16_nhwc": LC("odd_c_bf16_nhwc", 2, 7, 5, 60, 12, 6, "bf16", "nhwc", "gelu", 50),
+    "many_tiles_bf16_nhwc": LC("many_tiles_bf16_nhwc", 2, 23, 29, 128, 33, 12, "bf16", "nhwc",
+                               "relu", 100),
     "k1": LC("k1", 2, 5, 5, 16, 16, 1, "f32", "nhwc", "relu", 16),
     "one_position": LC("one_position", 4, 1, 1, 40, 12, 7, "f32", "nhwc", "gelu", 30),
     "rn50_stage1_reduce": CFG["rn50_stage1_reduce"].replace(N=2),
