@@ -68,9 +68,10 @@ def _load():
         lib.moce_oracle_coverage.argtypes = [I, I, P, D, P, P, P]
         lib.moce_oracle_backward.argtypes = [P, P, I, I, I, I, I, I, I, P, P, P, I, P, P, P, F, D,
                                              D, P, P, P, P, P, P]
+        lib.moce_oracle_dynamic_logits.argtypes = [P, I, I, I, I, I, I, I, P, P, P, P, P, P, P]
         for fn in (lib.moce_oracle_topk, lib.moce_oracle_pack, lib.moce_oracle_forward,
                    lib.moce_oracle_bruteforce_forward, lib.moce_oracle_coverage,
-                   lib.moce_oracle_backward):
+                   lib.moce_oracle_backward, lib.moce_oracle_dynamic_logits):
             fn.restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -311,3 +312,55 @@ class _use_library:
         global _lib
         _lib = self._saved
         return False
+
+
+def dynamic_logits(x: np.ndarray, layout: str, L, Wh, bh, V, Q):
+    """Eq. (dynamic): per-example logits L_e(X) = L_e + <q_e (.) h(z), v_c>, h(z) = ReLU(W_h z + b_h).
+
+    L [R, C], Wh [d, C], bh [d], V [C, d], Q [R, d]. Returns (h [N, d], Ldyn [N, R, C]), float64.
+    """
+    x = _c(x, np.float32)
+    if layout == "nhwc":
+        N, H, W, C = x.shape
+    else:
+        N, C, H, W = x.shape
+    L = _c(L, np.float32)
+    R = L.shape[0]
+    Wh = _c(Wh, np.float32)
+    d = Wh.shape[0]
+    h = np.empty((N, d), np.float64)
+    Ld = np.empty((N, R, C), np.float64)
+    st = _load().moce_oracle_dynamic_logits(_p(x), N, H, W, C, _LAYOUT[layout], R, d, _p(L), _p(Wh),
+                                            _p(_c(bh, np.float32)), _p(_c(V, np.float32)),
+                                            _p(_c(Q, np.float32)), _p(h), _p(Ld))
+    if st != OK:
+        raise OracleError(st, "dynamic_logits")
+    return h, Ld
+
+
+def dynamic_forward(x: np.ndarray, layout: str, L, Wh, bh, V, Q, k: int, W1, b1, w2, b2: float,
+                    tau_min: float, tau_max: float):
+    """The input-conditioned support variant (Sec. 5, Eq. dynamic), inference path.
+
+    Per example: the logits of Eq. (dynamic); S_e(X) = TopK(L_e(X), k) decided on the float32
+    values (the precision of the device path), in deployment order; U(X) the channels no
+    expert of that example selects; the gate reads z at S_e(X) and the weights use the selected
+    L_e(X) values (Eq. weights); then Eqs. (expert) and (res). Returns a dict: y, idx [N, R, k],
+    logits [N, R, k] (float32), resid (a list of N int32 arrays), h [N, d], Ldyn [N, R, C].
+    """
+    h, Ld = dynamic_logits(x, layout, L, Wh, bh, V, Q)
+    N, R, C = Ld.shape
+    ys, idxs, lgs, resids = [], [], [], []
+    for n in range(N):
+        Lf = Ld[n].astype(np.float32)
+        idx, lg = topk(Lf, k)
+        pidx, plog, resid = pack(idx, lg, C)
+        ys.append(forward(x[n:n + 1], layout, pidx, plog, resid, W1, b1, w2, b2, tau_min,
+                          tau_max))
+        idxs.append(pidx)
+        lgs.append(plog)
+        resids.append(resid)
+    y = np.concatenate(ys, axis=0) if ys else np.zeros((0,), np.float64)
+    return {"y": y, "idx": np.stack(idxs) if idxs else np.zeros((0, R, k), np.int32),
+            "logits": np.stack(lgs) if lgs else np.zeros((0, R, k), np.float32),
+            "resid": resids, "h": h, "Ldyn": Ld}

@@ -26,6 +26,11 @@
  *             values; no gradient through the indices): the gradients of a
  *             scalar loss with respect to x, the selected logits and the gate
  *             parameters, given dy, by the chain rule through the steps above
+ *   dynamic   Eq. (dynamic), input-conditioned support variant (Sec. 5): the
+ *             example's logits L_e(X) = L_e + <q_e (.) h(z), v_c> with the
+ *             router bottleneck h(z) = ReLU(W_h z + b_h); the per-example
+ *             TopK, U(X), gate and mixing then reuse the functions above with
+ *             that example's supports and logits
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - ties between equal logits order by ascending channel index; -0.0 and
@@ -627,5 +632,51 @@ int moce_oracle_backward(const float *x, const float *dy, int N, int H, int W, i
         }
     }
     free(z); free(u); free(hpre); free(a); free(da); free(dh); free(dz); free(aall);
+    return ORACLE_OK;
+}
+
+/*
+ * Eq. (dynamic): the input-conditioned routing logits of each example.
+ *   z = GAP(X) (Sec. 3.3), h(z) = ReLU(W_h z + b_h) in R^d,
+ *   L_e(X)_c = L_{e,c} + <q_e (.) h(z), v_c> = L_{e,c} + sum_j q_{e,j} h_j v_{c,j}.
+ * L [R][C] is the static routing matrix (row e = L_e), W_h [d][C] row-major,
+ * b_h [d], V [C][d] (row c = v_c), Q [R][d] (row e = q_e). Outputs, double:
+ * h_out [N][d] (optional) and Ldyn [N][R][C].
+ */
+int moce_oracle_dynamic_logits(const float *x, int N, int H, int W, int C, int layout, int R,
+                               int d, const float *L, const float *Wh, const float *bh,
+                               const float *V, const float *Q, double *h_out, double *Ldyn)
+{
+    if (N < 0 || H < 1 || W < 1 || C < 1 || R < 1 || d < 1 || (layout != 0 && layout != 1) ||
+        !L || !Wh || !bh || !V || !Q || !Ldyn)
+        return ORACLE_BAD_ARG;
+    double *z = (double *)malloc(sizeof(double) * (size_t)C * (N > 0 ? N : 1));
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!z || !h) {
+        free(z);
+        free(h);
+        return ORACLE_NO_MEMORY;
+    }
+    moce_oracle_pool(x, N, H, W, C, layout, z);
+    for (int n = 0; n < N; ++n) {
+        const double *zn = z + (size_t)n * C;
+        for (int j = 0; j < d; ++j) {
+            double s = (double)bh[j];
+            for (int c = 0; c < C; ++c)
+                s += (double)Wh[(size_t)j * C + c] * zn[c];
+            h[j] = s > 0.0 ? s : 0.0;
+            if (h_out)
+                h_out[(size_t)n * d + j] = h[j];
+        }
+        for (int e = 0; e < R; ++e)
+            for (int c = 0; c < C; ++c) {
+                double off = 0.0;
+                for (int j = 0; j < d; ++j)
+                    off += (double)Q[(size_t)e * d + j] * h[j] * (double)V[(size_t)c * d + j];
+                Ldyn[((size_t)n * R + e) * C + c] = (double)L[(size_t)e * C + c] + off;
+            }
+    }
+    free(z);
+    free(h);
     return ORACLE_OK;
 }

@@ -60,6 +60,16 @@ MUTANTS = {
                                  "du += (double)W1[(size_t)i * k + j] * dh[j];"),
     "backward_residual_not_divided": ("const double d = (double)dy[x_at(layout, n, p, R, HW, E)] / (double)n_resid;",
                                       "const double d = (double)dy[x_at(layout, n, p, R, HW, E)];"),
+    "dynamic_relu_dropped": ("h[j] = s > 0.0 ? s : 0.0;\n            if (h_out)",
+                             "h[j] = s;\n            if (h_out)"),
+    "dynamic_bias_dropped": ("double s = (double)bh[j];", "double s = 0.0;"),
+    "dynamic_V_transposed": ("(double)V[(size_t)c * d + j];", "(double)V[(size_t)j * C + c];"),
+    "dynamic_Wh_transposed": ("s += (double)Wh[(size_t)j * C + c] * zn[c];",
+                              "s += (double)Wh[(size_t)c * d + j] * zn[c];"),
+    "dynamic_Q_uses_channel": ("off += (double)Q[(size_t)e * d + j] * h[j]",
+                               "off += (double)Q[(size_t)(c % R) * d + j] * h[j]"),
+    "dynamic_offset_sign": ("Ldyn[((size_t)n * R + e) * C + c] = (double)L[(size_t)e * C + c] + off;",
+                            "Ldyn[((size_t)n * R + e) * C + c] = (double)L[(size_t)e * C + c] - off;"),
     "coverage_grad_softmax_jacobian_dot_dropped": ("p[(size_t)e * C + c] * (g[c] - dot) / (double)R;",
                                                    "p[(size_t)e * C + c] * g[c] / (double)R;"),
 }
@@ -88,6 +98,11 @@ PIN_CHECKS = [
     pins.test_coverage_equals_numpy_definition_and_finite_differences,
     lambda: pins.test_backward_equals_central_differences("nhwc"),
     pins.test_backward_constant_temperature_is_the_transposed_linear_map,
+    lambda: pins.test_dynamic_offset_vanishes("h"),
+    pins.test_dynamic_single_coupling_lands_on_one_expert_and_channel,
+    lambda: pins.test_dynamic_router_reads_the_pooled_descriptor("nhwc"),
+    pins.test_dynamic_offset_has_rank_at_most_d_and_is_bilinear,
+    pins.test_dynamic_supports_follow_each_example,
 ]
 
 

@@ -479,3 +479,145 @@ def test_backward_is_linear_in_dy():
     for name in ("dx", "dlogit", "dW1", "db1", "dw2"):
         want = g1[name] + g2[name]
         np.testing.assert_allclose(g3[name], want, rtol=0, atol=1e-6 * np.abs(want).max())
+
+
+# ---------------------------------------------------------------- input-conditioned supports
+# Eq. (dynamic): L_e(X)_c = L_{e,c} + <q_e (.) h(z), v_c>, h(z) = ReLU(W_h z + b_h).
+
+
+def _dyn_setup(seed=0, N=2, H=3, W=5, C=20, R=6, d=4, layout="nhwc"):
+    rng = np.random.default_rng(seed)
+    shape = (N, H, W, C) if layout == "nhwc" else (N, C, H, W)
+    x = rng.standard_normal(shape).astype(np.float32)
+    L = rng.standard_normal((R, C)).astype(np.float32)
+    Wh = (rng.standard_normal((d, C)) / np.sqrt(C)).astype(np.float32)
+    bh = (0.5 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    V = rng.standard_normal((C, d)).astype(np.float32)
+    Q = rng.standard_normal((R, d)).astype(np.float32)
+    return x, L, Wh, bh, V, Q
+
+
+@pytest.mark.parametrize("zero", ["Q", "V", "h"])
+def test_dynamic_offset_vanishes(zero):
+    """No router signal (q = 0, v = 0, or h = ReLU(negative) = 0): L(X) is the static L exactly."""
+    x, L, Wh, bh, V, Q = _dyn_setup(1)
+    if zero == "Q":
+        Q[:] = 0
+    elif zero == "V":
+        V[:] = 0
+    else:
+        Wh[:] = 0
+        bh[:] = -1.0
+    h, Ld = oracle.dynamic_logits(x, "nhwc", L, Wh, bh, V, Q)
+    for n in range(x.shape[0]):
+        assert np.array_equal(Ld[n], L.astype(np.float64))
+    if zero == "h":
+        assert np.all(h == 0.0)
+
+
+def test_dynamic_single_coupling_lands_on_one_expert_and_channel():
+    """One router unit j0 active (h = b at j0 only), q_e nonzero only at (e0, j0), v_c only at
+    (c0, j0): the offset is q * b * v at exactly (e0, c0)."""
+    x, L, Wh, bh, V, Q = _dyn_setup(2, d=3)
+    Wh[:] = 0
+    bh[:] = [0.0, 1.5, 0.0]
+    Q[:] = 0
+    V[:] = 0
+    e0, c0 = 4, 13
+    Q[e0, 1] = -2.0
+    V[c0, 1] = 0.75
+    Q[1, 0] = 9.0  # couples through unit 0, which is inactive
+    V[3, 2] = 9.0  # unit 2 is inactive too
+    h, Ld = oracle.dynamic_logits(x, "nhwc", L, Wh, bh, V, Q)
+    want = L.astype(np.float64).copy()
+    want[e0, c0] += -2.0 * 1.5 * 0.75
+    for n in range(x.shape[0]):
+        np.testing.assert_array_equal(Ld[n], want)
+        np.testing.assert_array_equal(h[n], [0.0, 1.5, 0.0])
+
+
+@pytest.mark.parametrize("layout", ["nhwc", "nchw"])
+def test_dynamic_router_reads_the_pooled_descriptor(layout):
+    """x constant over positions (x[n,p,c] = s_{n,c}) gives z = s; a router row that reads one
+    channel c1 gives h_j = ReLU(w s_{c1} + b_j) for W_h [d][C] with row j = unit j."""
+    N, H, W, C, R, d = 3, 2, 3, 10, 4, 2
+    rng = np.random.default_rng(3)
+    s = rng.standard_normal((N, C)).astype(np.float32)
+    x = np.broadcast_to(s[:, None, None, :], (N, H, W, C)).astype(np.float32)
+    if layout == "nchw":
+        x = np.ascontiguousarray(x.transpose(0, 3, 1, 2))
+    L = np.zeros((R, C), np.float32)
+    Wh = np.zeros((d, C), np.float32)
+    Wh[1, 7] = 2.0            # unit 1 reads channel 7
+    bh = np.array([-5.0, 0.25], np.float32)
+    V = np.zeros((C, d), np.float32)
+    V[:, 1] = np.arange(C, dtype=np.float32)
+    Q = np.zeros((R, d), np.float32)
+    Q[:, 1] = 1.0
+    h, Ld = oracle.dynamic_logits(x, layout, L, Wh, bh, V, Q)
+    for n in range(N):
+        hv = max(0.0, 2.0 * float(s[n, 7]) + 0.25)
+        np.testing.assert_allclose(h[n], [0.0, hv], rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(Ld[n], np.tile(hv * np.arange(C), (R, 1)), rtol=1e-12,
+                                   atol=1e-12)
+
+
+def test_dynamic_offset_has_rank_at_most_d_and_is_bilinear():
+    x, L, Wh, bh, V, Q = _dyn_setup(4, C=24, R=10, d=3)
+    _, Ld = oracle.dynamic_logits(x, "nhwc", L, Wh, bh, V, Q)
+    for n in range(x.shape[0]):
+        sv = np.linalg.svd(Ld[n] - L, compute_uv=False)
+        assert sv[3] <= 1e-9 * sv[0]
+    # powers of two keep the scaled float32 parameters exact
+    _, Ld2 = oracle.dynamic_logits(x, "nhwc", L, Wh, bh, 2.0 * V, 4.0 * Q)
+    np.testing.assert_allclose(Ld2 - L, 8.0 * (Ld - L), rtol=1e-12, atol=1e-12)
+
+
+def test_dynamic_forward_without_router_signal_is_the_static_layer():
+    """q = 0: every example selects TopK(L) and the layer is the static forward (Sec. 5: the
+    variant replaces only the support of Eq. support)."""
+    x, L, Wh, bh, V, Q = _dyn_setup(5, N=3, C=16, R=5)
+    Q[:] = 0
+    k = 4
+    rng = np.random.default_rng(6)
+    W1 = (rng.standard_normal((k, k)) / 2).astype(np.float32)
+    b1 = rng.standard_normal(k).astype(np.float32)
+    w2 = rng.standard_normal(k).astype(np.float32)
+    out = oracle.dynamic_forward(x, "nhwc", L, Wh, bh, V, Q, k, W1, b1, w2, 0.3, 0.2, 6.0)
+    pidx, plog, resid = oracle.pack(*oracle.topk(L, k), 16)
+    ys = oracle.forward(x, "nhwc", pidx, plog, resid, W1, b1, w2, 0.3, 0.2, 6.0)
+    np.testing.assert_array_equal(out["y"], ys)
+    for n in range(3):
+        assert np.array_equal(out["idx"][n], pidx) and np.array_equal(out["resid"][n], resid)
+
+
+def test_dynamic_supports_follow_each_example():
+    """A strong router term moves each example's supports toward the channels its own
+    descriptor favours; U(X) is the complement of that example's union of supports."""
+    N, H, W, C, R, d, k = 2, 2, 2, 12, 3, 1, 2
+    x = np.zeros((N, H, W, C), np.float32)
+    x[0, :, :, 0] = 1.0       # example 0 pools to channel 0 only
+    x[1, :, :, 1] = 1.0       # example 1 pools to channel 1 only
+    L = np.zeros((R, C), np.float32)
+    L[:, 2:] = -np.arange(1, C - 1, dtype=np.float32) * 0.01  # static order: 0, 1 tie, then 2, 3, ...
+    Wh = np.zeros((d, C), np.float32)
+    Wh[0, 0] = 1.0            # h = ReLU(z_0): 1 for example 0, 0 for example 1
+    bh = np.zeros(d, np.float32)
+    V = np.zeros((C, d), np.float32)
+    V[5, 0] = 10.0
+    V[6, 0] = 9.0             # router pulls channels 5 and 6 up for example 0
+    Q = np.ones((R, d), np.float32)
+    W1 = np.zeros((k, k), np.float32)
+    b1 = np.zeros(k, np.float32)
+    w2 = np.zeros(k, np.float32)
+    out = oracle.dynamic_forward(x, "nhwc", L, Wh, bh, V, Q, k, W1, b1, w2, 0.0, 1.0, 1.0)
+    assert out["idx"][0].tolist() == [[5, 6]] * R
+    assert out["idx"][1].tolist() == [[0, 1]] * R
+    assert out["resid"][0].tolist() == [c for c in range(C) if c not in (5, 6)]
+    assert out["resid"][1].tolist() == list(range(2, C))
+    # tau = 1 (tau_min = tau_max): a = softmax of the example's selected logits
+    a0 = sp_softmax(np.array([10.0, 9.0]) + L[0, [5, 6]])
+    np.testing.assert_allclose(out["y"][0, 0, 0, 0], 0.0, atol=0)  # x is 0 on channels 5 and 6
+    np.testing.assert_allclose(out["y"][1, 0, 0, :R], np.full(R, sp_softmax([0.0, 0.0])[1]),
+                               rtol=1e-12)
+    assert a0[0] > a0[1]
