@@ -664,7 +664,7 @@ int moce_oracle_dynamic_logits(const float *x, int N, int H, int W, int C, int l
             double s = (double)bh[j];
             for (int c = 0; c < C; ++c)
                 s += (double)Wh[(size_t)j * C + c] * zn[c];
-            h[j] = s > 0.0 ? s : 0.0;
+            h[j] = (s > 0.0) ? s : 0.0; /* ReLU of the router bottleneck */
             if (h_out)
                 h_out[(size_t)n * d + j] = h[j];
         }

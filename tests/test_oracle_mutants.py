@@ -60,8 +60,7 @@ MUTANTS = {
                                  "du += (double)W1[(size_t)i * k + j] * dh[j];"),
     "backward_residual_not_divided": ("const double d = (double)dy[x_at(layout, n, p, R, HW, E)] / (double)n_resid;",
                                       "const double d = (double)dy[x_at(layout, n, p, R, HW, E)];"),
-    "dynamic_relu_dropped": ("h[j] = s > 0.0 ? s : 0.0;\n            if (h_out)",
-                             "h[j] = s;\n            if (h_out)"),
+    "dynamic_relu_dropped": ("h[j] = (s > 0.0) ? s : 0.0; /* ReLU", "h[j] = s; /* ReLU"),
     "dynamic_bias_dropped": ("double s = (double)bh[j];", "double s = 0.0;"),
     "dynamic_V_transposed": ("(double)V[(size_t)c * d + j];", "(double)V[(size_t)j * C + c];"),
     "dynamic_Wh_transposed": ("s += (double)Wh[(size_t)j * C + c] * zn[c];",
