@@ -238,6 +238,83 @@ moce_status_t moce_forward_noalloc(const void *x, int N, int H, int W, int C_in,
                                    float tau_min, float tau_max, void *y, moce_stream_t stream);
 
 /*
+ * Routed mix and residual expert alone, Eq. (expert) and Eq. (res), from
+ * precomputed weights mix_w [N][C_out][k] (moce_gate's output).
+ *   n_resid_per_example == NULL: shared supports, sup_idx [C_out][k] and
+ *     resid_idx [C_in] with n_resid entries (as moce_forward);
+ *   otherwise per-example supports, sup_idx [N][C_out][k], resid_idx
+ *     [N][C_in] and n_resid_per_example [N] (device), as written by
+ *     moce_dynamic_supports; n_resid is ignored.
+ * ws: a forward workspace (moce_workspace_bytes). Asynchronous.
+ */
+moce_status_t moce_mix(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                       moce_dtype_t dtype, moce_layout_t layout, const int32_t *sup_idx,
+                       const float *mix_w, const int32_t *resid_idx, int n_resid,
+                       const int32_t *n_resid_per_example, void *y, void *ws, size_t ws_bytes,
+                       moce_stream_t stream);
+
+/*
+ * Input-conditioned supports, Eq. (dynamic) (the variant of Sec. 5; the
+ * inference path: deterministic hard per-example TopK, no noise). A router
+ * reads the whole pooled descriptor z = GAP(X) and adds a rank-d offset to
+ * the static routing matrix; each example then selects its own supports:
+ *   h(z)      = ReLU(W_h z + b_h)                          in R^d
+ *   L_e(X)_c  = L_{e,c} + sum_j q_{e,j} h_j v_{c,j}        every e, c
+ *   S_e(X)    = TopK(L_e(X), k), in deployment order (descending L_e(X),
+ *               equal values by ascending channel), decided in fp32
+ *   U(X)      = the channels no S_e(X) selects, ascending
+ * and the layer of moce_forward runs with these supports: the gate reads z
+ * at S_e(X) (Sec. 3.3 ordering) and the weights use the selected L_e(X)
+ * values in place of L_{e,i} (Eq. (weights)).
+ *   logits  device fp32 [C_out][C_in]: the static routing matrix L
+ *   Wh      device fp32 [d][C_in] (row j = router unit j), bh [d]
+ *   V       device fp32 [C_in][d] (row c = channel embedding v_c)
+ *   Q       device fp32 [C_out][d] (row e = expert embedding q_e)
+ * (2 C_in d + d + C_out d router parameters, as the paper counts them.)
+ * C_in <= 16384 (TopK sorts a row in shared memory), 1 <= d <= 4096.
+ * Non-finite logits give unspecified (but in-range) supports.
+ *
+ * moce_dynamic_workspace_bytes: device workspace of the dynamic calls
+ * (256-byte aligned, no initialisation needed); 0 for unsupported shapes.
+ * Its routing buffers come first and do not depend on H and W, so
+ * moce_dynamic_supports accepts the workspace of any H, W.
+ *
+ * moce_dynamic_supports: from pooled descriptors z [N][C_in] (moce_pool)
+ * to the per-example supports sup_idx / sup_logits [N][C_out][k], U(X) in
+ * resid_idx [N][C_in] (the first n_resid[n] entries of row n) and
+ * n_resid [N] (all device, int32 / fp32). Asynchronous.
+ *
+ * moce_forward_supports: the layer with given per-example supports (as
+ * moce_dynamic_supports writes them): pool, gate and mix. ws: a forward
+ * workspace (moce_workspace_bytes). Asynchronous.
+ *
+ * moce_forward_dynamic: the whole variant: pool, router, TopK, U(X), gate and
+ * mix. sup_idx, sup_logits, n_resid: optional device outputs (NULL: kept in
+ * the workspace). Asynchronous.
+ */
+size_t moce_dynamic_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k, int d);
+moce_status_t moce_dynamic_supports(const float *z, int N, int C_in, int C_out, int k, int d,
+                                    const float *logits, const float *Wh, const float *bh,
+                                    const float *V, const float *Q, int32_t *sup_idx,
+                                    float *sup_logits, int32_t *resid_idx, int32_t *n_resid,
+                                    void *ws, size_t ws_bytes, moce_stream_t stream);
+moce_status_t moce_forward_supports(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                    moce_dtype_t dtype, moce_layout_t layout,
+                                    const int32_t *sup_idx, const float *sup_logits,
+                                    const int32_t *resid_idx, const int32_t *n_resid,
+                                    const float *W1, const float *b1, const float *w2,
+                                    const float *b2, float tau_min, float tau_max, void *y,
+                                    void *ws, size_t ws_bytes, moce_stream_t stream);
+moce_status_t moce_forward_dynamic(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                   int d, moce_dtype_t dtype, moce_layout_t layout,
+                                   const float *logits, const float *Wh, const float *bh,
+                                   const float *V, const float *Q, const float *W1,
+                                   const float *b1, const float *w2, const float *b2,
+                                   float tau_min, float tau_max, void *y, int32_t *sup_idx,
+                                   float *sup_logits, int32_t *n_resid, void *ws, size_t ws_bytes,
+                                   moce_stream_t stream);
+
+/*
  * SYNCHRONOUS: waits for `stream`, then reads the device error word that the
  * last moce_forward_noalloc on the current device left in the scratch array.
  * MOCE_OK, MOCE_ERR_TIMEOUT (a bounded wait of that forward gave up; its y is

@@ -21,7 +21,7 @@ LIB = os.path.join(BUILD, "libmoce.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["moce_api.cu", "moce_pack.cu", "moce_pool.cu", "moce_gate.cu", "moce_mix.cu",
            "moce_mix_wide.cu", "moce_noalloc.cu", "moce_stream.cu", "moce_train.cu",
-           "moce_backward.cu"]
+           "moce_backward.cu", "moce_dynamic.cu"]
 
 
 def nvcc() -> str:

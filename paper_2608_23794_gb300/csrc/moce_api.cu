@@ -276,6 +276,155 @@ moce_status_t moce_coverage_loss(const float *logits, int C_in, int C_out, float
                                        reinterpret_cast<cudaStream_t>(stream)));
 }
 
+moce_status_t moce_mix(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                       moce_dtype_t dtype, moce_layout_t layout, const int32_t *sup_idx,
+                       const float *mix_w, const int32_t *resid_idx, int n_resid,
+                       const int32_t *n_resid_per_example, void *y, void *ws, size_t ws_bytes,
+                       moce_stream_t stream) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout))
+        return MOCE_ERR_INVALID_VALUE;
+    const bool per = n_resid_per_example != nullptr;
+    if (!per && (n_resid < 0 || n_resid > C_in || (n_resid > 0 && !resid_idx)))
+        return MOCE_ERR_INVALID_VALUE;
+    if (N == 0 || H * W == 0) return MOCE_OK;
+    if (!x || !sup_idx || !mix_w || !y || !ws || (per && !resid_idx)) return MOCE_ERR_INVALID_VALUE;
+    const WsLayout L = ws_layout(N, H * W, C_in, C_out, k);
+    if (ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255u)) return MOCE_ERR_INVALID_VALUE;
+    PerExample pe;
+    if (per) {
+        pe.sup_stride = (size_t)C_out * k;
+        pe.resid_stride = (size_t)C_in;
+        pe.nUa = n_resid_per_example;
+    }
+    unsigned char *wsb = static_cast<unsigned char *>(ws);
+    return cuda_status(launch_mix(x, N, H * W, C_in, C_out, k, dtype, layout, sup_idx, mix_w,
+                                  resid_idx, per ? 0 : n_resid, y,
+                                  reinterpret_cast<uint32_t *>(wsb + L.ctrl),
+                                  reinterpret_cast<cudaStream_t>(stream), pe));
+}
+
+static bool dyn_shape_ok(int N, int H, int W, int C_in, int C_out, int k, int d) {
+    return shape_ok(N, H, W, C_in, C_out, k) && d >= 1 && d <= 4096 &&
+           (long long)N * C_out <= (1ll << 31) - 1 &&
+           (long long)N * C_out * C_in <= (1ll << 40);
+}
+
+size_t moce_dynamic_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k, int d) {
+    if (!dyn_shape_ok(N, H, W, C_in, C_out, k, d) || !dynamic_supported(C_in)) return 0;
+    return dyn_layout(N, H * W, C_in, C_out, k, d).total;
+}
+
+moce_status_t moce_dynamic_supports(const float *z, int N, int C_in, int C_out, int k, int d,
+                                    const float *logits, const float *Wh, const float *bh,
+                                    const float *V, const float *Q, int32_t *sup_idx,
+                                    float *sup_logits, int32_t *resid_idx, int32_t *n_resid,
+                                    void *ws, size_t ws_bytes, moce_stream_t stream) {
+    if (!dyn_shape_ok(N, 1, 1, C_in, C_out, k, d)) return MOCE_ERR_INVALID_VALUE;
+    if (!dynamic_supported(C_in)) return MOCE_ERR_UNSUPPORTED;
+    if (N == 0) return MOCE_OK;
+    if (!z || !logits || !Wh || !bh || !V || !Q || !sup_idx || !sup_logits || !resid_idx ||
+        !n_resid || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    const DynLayout D = dyn_layout(N, 1, C_in, C_out, k, d);
+    if (ws_bytes < D.routing || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MOCE_ERR_INVALID_VALUE;
+    unsigned char *wsb = static_cast<unsigned char *>(ws);
+    return cuda_status(launch_dynamic_supports(
+        z, N, C_in, C_out, k, d, logits, Wh, bh, V, Q, reinterpret_cast<float *>(wsb + D.h),
+        reinterpret_cast<float *>(wsb + D.Ld), sup_idx, sup_logits, resid_idx, n_resid,
+        reinterpret_cast<uint32_t *>(wsb + D.err), reinterpret_cast<cudaStream_t>(stream)));
+}
+
+// Gate and mix with per-example supports; z already pooled at L.z of wsf.
+static cudaError_t run_with_supports(const void *x, int N, int HW, int C, int R, int k,
+                                     moce_dtype_t dt, moce_layout_t lay, const int32_t *sidx,
+                                     const float *slog, const int32_t *resid, const int32_t *nU,
+                                     const float *W1, const float *b1, const float *w2,
+                                     const float *b2, float tmin, float tmax, void *y,
+                                     const WsLayout &L, unsigned char *wsf, cudaStream_t s) {
+    float *z = reinterpret_cast<float *>(wsf + L.z);
+    float *tau = reinterpret_cast<float *>(wsf + L.tau);
+    float *a = reinterpret_cast<float *>(wsf + L.a);
+    cudaError_t err = launch_gate(z, N, C, R, k, sidx, slog, W1, b1, w2, b2, tmin, tmax, tau, a, s,
+                                  (size_t)R * k);
+    if (err != cudaSuccess) return err;
+    PerExample pe;
+    pe.sup_stride = (size_t)R * k;
+    pe.resid_stride = (size_t)C;
+    pe.nUa = nU;
+    return launch_mix(x, N, HW, C, R, k, dt, lay, sidx, a, resid, 0, y,
+                      reinterpret_cast<uint32_t *>(wsf + L.ctrl), s, pe);
+}
+
+moce_status_t moce_forward_supports(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                    moce_dtype_t dtype, moce_layout_t layout,
+                                    const int32_t *sup_idx, const float *sup_logits,
+                                    const int32_t *resid_idx, const int32_t *n_resid,
+                                    const float *W1, const float *b1, const float *w2,
+                                    const float *b2, float tau_min, float tau_max, void *y,
+                                    void *ws, size_t ws_bytes, moce_stream_t stream) {
+    if (!shape_ok(N, H, W, C_in, C_out, k) || !dtype_ok(dtype) || !layout_ok(layout) ||
+        !tau_ok(tau_min, tau_max))
+        return MOCE_ERR_INVALID_VALUE;
+    const int HW = H * W;
+    if (N == 0 || HW == 0) return MOCE_OK;
+    if (!x || !sup_idx || !sup_logits || !resid_idx || !n_resid || !W1 || !b1 || !w2 || !b2 ||
+        !y || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    const WsLayout L = ws_layout(N, HW, C_in, C_out, k);
+    if (ws_bytes < L.total || (reinterpret_cast<uintptr_t>(ws) & 255u)) return MOCE_ERR_INVALID_VALUE;
+    if (gate_smem_bytes(k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    unsigned char *wsb = static_cast<unsigned char *>(ws);
+    cudaError_t err = launch_pool(x, N, HW, C_in, dtype, layout,
+                                  reinterpret_cast<float *>(wsb + L.z), L, wsb, s);
+    if (err == cudaSuccess)
+        err = run_with_supports(x, N, HW, C_in, C_out, k, dtype, layout, sup_idx, sup_logits,
+                                resid_idx, n_resid, W1, b1, w2, b2, tau_min, tau_max, y, L, wsb, s);
+    return cuda_status(err);
+}
+
+moce_status_t moce_forward_dynamic(const void *x, int N, int H, int W, int C_in, int C_out, int k,
+                                   int d, moce_dtype_t dtype, moce_layout_t layout,
+                                   const float *logits, const float *Wh, const float *bh,
+                                   const float *V, const float *Q, const float *W1,
+                                   const float *b1, const float *w2, const float *b2,
+                                   float tau_min, float tau_max, void *y, int32_t *sup_idx,
+                                   float *sup_logits, int32_t *n_resid, void *ws, size_t ws_bytes,
+                                   moce_stream_t stream) {
+    if (!dyn_shape_ok(N, H, W, C_in, C_out, k, d) || !dtype_ok(dtype) || !layout_ok(layout) ||
+        !tau_ok(tau_min, tau_max))
+        return MOCE_ERR_INVALID_VALUE;
+    if (!dynamic_supported(C_in)) return MOCE_ERR_UNSUPPORTED;
+    const int HW = H * W;
+    if (N == 0 || HW == 0) return MOCE_OK;
+    if (!x || !logits || !Wh || !bh || !V || !Q || !W1 || !b1 || !w2 || !b2 || !y || !ws)
+        return MOCE_ERR_INVALID_VALUE;
+    const DynLayout D = dyn_layout(N, HW, C_in, C_out, k, d);
+    if (ws_bytes < D.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MOCE_ERR_INVALID_VALUE;
+    if (gate_smem_bytes(k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    unsigned char *wsb = static_cast<unsigned char *>(ws);
+    unsigned char *wsf = wsb + D.fwd_off;
+    const WsLayout &L = D.fwd;
+    float *z = reinterpret_cast<float *>(wsf + L.z);
+    int32_t *sidx = sup_idx ? sup_idx : reinterpret_cast<int32_t *>(wsb + D.sidx);
+    float *slog = sup_logits ? sup_logits : reinterpret_cast<float *>(wsb + D.slog);
+    int32_t *nU = n_resid ? n_resid : reinterpret_cast<int32_t *>(wsb + D.nU);
+    int32_t *resid = reinterpret_cast<int32_t *>(wsb + D.resid);
+    cudaError_t err = launch_pool(x, N, HW, C_in, dtype, layout, z, L, wsf, s);
+    if (err == cudaSuccess)
+        err = launch_dynamic_supports(z, N, C_in, C_out, k, d, logits, Wh, bh, V, Q,
+                                      reinterpret_cast<float *>(wsb + D.h),
+                                      reinterpret_cast<float *>(wsb + D.Ld), sidx, slog, resid, nU,
+                                      reinterpret_cast<uint32_t *>(wsb + D.err), s);
+    if (err == cudaSuccess)
+        err = run_with_supports(x, N, HW, C_in, C_out, k, dtype, layout, sidx, slog, resid, nU, W1,
+                                b1, w2, b2, tau_min, tau_max, y, L, wsf, s);
+    return cuda_status(err);
+}
+
 size_t moce_backward_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k) {
     if (!shape_ok(N, H, W, C_in, C_out, k)) return 0;
     return backward_ws_bytes(N, H * W, C_in, C_out, k);

@@ -22,10 +22,11 @@ __global__ void __launch_bounds__(kThreads) gate_kernel(
     const float *__restrict__ z, int C, int R, int k, const int32_t *__restrict__ pidx,
     const float *__restrict__ plog, const float *__restrict__ W1, const float *__restrict__ b1,
     const float *__restrict__ w2, const float *__restrict__ b2, float tmin, float tmax,
-    float *__restrict__ tau, float *__restrict__ a) {
+    float *__restrict__ tau, float *__restrict__ a, size_t sup_stride) {
     extern __shared__ __align__(16) float gsm[];
-    gate_block(gsm, blockIdx.y, blockIdx.x * GE, z, C, R, k, pidx, plog, W1, b1, w2, b2, tmin, tmax,
-               tau, a);
+    const size_t so = (size_t)blockIdx.y * sup_stride;  // per-example supports (0: shared)
+    gate_block(gsm, blockIdx.y, blockIdx.x * GE, z, C, R, k, pidx + so, plog + so, W1, b1, w2, b2,
+               tmin, tmax, tau, a);
 }
 
 constexpr int kTE = 64;        // experts per tiled-gate CTA
@@ -51,8 +52,10 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
     const float *__restrict__ z, int C, int R, const int32_t *__restrict__ pidx,
     const float *__restrict__ plog, const float *__restrict__ W1, const float *__restrict__ b1,
     const float *__restrict__ w2, const float *__restrict__ b2, float tmin, float tmax,
-    float *__restrict__ tau, float *__restrict__ a) {
+    float *__restrict__ tau, float *__restrict__ a, size_t sup_stride) {
     constexpr int k = 16 * TN;
+    pidx += (size_t)blockIdx.y * sup_stride;  // per-example supports (0: shared)
+    plog += (size_t)blockIdx.y * sup_stride;
     extern __shared__ __align__(16) float tsm[];
     const int KC = tiled_kc(k);
     float *Ut = tsm;                      // [k][kUS]: Ut[i][el] = z[n, S_(e0 + el)][i]
@@ -201,7 +204,7 @@ template <int TN>
 cudaError_t launch_tiled_gate(const float *z, int N, int C, int R, const int32_t *pidx,
                               const float *plog, const float *W1, const float *b1,
                               const float *w2, const float *b2, float tmin, float tmax,
-                              float *tau, float *a, cudaStream_t s) {
+                              float *tau, float *a, size_t ss, cudaStream_t s) {
     constexpr int k = 16 * TN;
     const size_t smem = tiled_smem(k, C);
     cudaError_t err = cudaFuncSetAttribute(gate_tiled_kernel<TN>,
@@ -209,7 +212,7 @@ cudaError_t launch_tiled_gate(const float *z, int N, int C, int R, const int32_t
     if (err != cudaSuccess) return err;
     const dim3 grid((R + kTE - 1) / kTE, N);
     gate_tiled_kernel<TN><<<grid, 256, smem, s>>>(z, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax,
-                                                  tau, a);
+                                                  tau, a, ss);
     return cudaGetLastError();
 }
 
@@ -218,20 +221,20 @@ cudaError_t launch_tiled_gate(const float *z, int N, int C, int R, const int32_t
 cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_t *pidx,
                         const float *plog, const float *W1, const float *b1, const float *w2,
                         const float *b2, float tmin, float tmax, float *tau, float *a,
-                        cudaStream_t s) {
+                        cudaStream_t s, size_t ss) {
     if (N == 0) return cudaSuccess;
     // the tiled kernel reads W1 rows as float4
     const bool w1v = (reinterpret_cast<uintptr_t>(W1) & 15u) == 0 &&
-                     (reinterpret_cast<uintptr_t>(pidx) & 15u) == 0;
+                     (reinterpret_cast<uintptr_t>(pidx) & 15u) == 0 && ss % 4 == 0;
     if (w1v && k >= 32 && tiled_smem(k, C) <= 227 * 1024) {
         switch (k) {
-        case 32: return launch_tiled_gate<2>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 64: return launch_tiled_gate<4>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 96: return launch_tiled_gate<6>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 128: return launch_tiled_gate<8>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 192: return launch_tiled_gate<12>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 256: return launch_tiled_gate<16>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
-        case 384: return launch_tiled_gate<24>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, s);
+        case 32: return launch_tiled_gate<2>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 64: return launch_tiled_gate<4>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 96: return launch_tiled_gate<6>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 128: return launch_tiled_gate<8>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 192: return launch_tiled_gate<12>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 256: return launch_tiled_gate<16>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
+        case 384: return launch_tiled_gate<24>(z, N, C, R, pidx, plog, W1, b1, w2, b2, tmin, tmax, tau, a, ss, s);
         default: break;
         }
     }
@@ -243,7 +246,7 @@ cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_
     }
     const dim3 grid((R + GE - 1) / GE, N);
     gate_kernel<<<grid, kThreads, smem, s>>>(z, C, R, k, pidx, plog, W1, b1, w2, b2, tmin, tmax,
-                                             tau, a);
+                                             tau, a, ss);
     return cudaGetLastError();
 }
 

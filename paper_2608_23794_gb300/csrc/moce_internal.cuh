@@ -121,15 +121,26 @@ cudaError_t launch_pack(int C, int R, int k, const int32_t *idx, const float *lg
 cudaError_t launch_pool(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay,
                         float *z, const WsLayout &L, unsigned char *ws, cudaStream_t s);
 
+// sup_stride: elements between two examples' supports in pidx / plog (0:
+// every example shares one set of supports).
 cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_t *pidx,
                         const float *plog, const float *W1, const float *b1, const float *w2,
                         const float *b2, float tmin, float tmax, float *tau, float *a,
-                        cudaStream_t s);
+                        cudaStream_t s, size_t sup_stride = 0);
+
+// Per-example supports of the mixing kernels: example n reads its supports
+// at pidx + n sup_stride, its U at resid + n resid_stride and |U| at nUa[n]
+// (a device array; when nUa is null every example has the scalar nU).
+struct PerExample {
+    size_t sup_stride = 0, resid_stride = 0;
+    const int32_t *nUa = nullptr;
+};
 
 // ctrl: the workspace control words (bounded waits report MOCE_ERR_TIMEOUT there).
 cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
                        moce_layout_t lay, const int32_t *pidx, const float *a,
-                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s);
+                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s,
+                       const PerExample &pe = PerExample());
 
 // Mixing kernel for wide layers (moce_mix_wide.cu): NHWC bf16, C % 8 == 0,
 // x 16-byte aligned.
@@ -156,6 +167,27 @@ cudaError_t launch_backward(const void *x, const void *dy, int N, int HW, int C,
                             const float *b1, const float *w2, const float *b2, float tmin,
                             float tmax, float *dx, float *dlogit, float *dW1, float *db1,
                             float *dw2, float *db2, unsigned char *ws, cudaStream_t s);
+
+// Input-conditioned supports (moce_dynamic.cu). Workspace: the routing
+// buffers first (their offsets depend on N, C, R, k, d only), then a forward
+// workspace (ws_layout) at fwd_off.
+struct DynLayout {
+    size_t err = 0, h = 0, Ld = 0, sidx = 0, slog = 0, resid = 0, nU = 0;
+    size_t routing = 0;  // bytes of the routing buffers
+    size_t fwd_off = 0;
+    WsLayout fwd;
+    size_t total = 0;
+};
+DynLayout dyn_layout(int N, int HW, int C, int R, int k, int d);
+bool dynamic_supported(int C);
+// From pooled descriptors z [N][C]: h [N][d], the logits Ld [N][R][C], the
+// per-example supports sidx / slog [N][R][k] (deployment order), U(X) in
+// resid [N][C] (ascending) and |U(X)| in nU [N]. err: TopK's non-finite flag.
+cudaError_t launch_dynamic_supports(const float *z, int N, int C, int R, int k, int d,
+                                    const float *L, const float *Wh, const float *bh,
+                                    const float *V, const float *Q, float *h, float *Ld,
+                                    int32_t *sidx, float *slog, int32_t *resid, int32_t *nU,
+                                    uint32_t *err, cudaStream_t s);
 
 cudaError_t launch_stream(const uint16_t *x, int N, int HW, int C, int R, int k,
                           const int32_t *pidx, const float *plog, const int32_t *resid, int nU,

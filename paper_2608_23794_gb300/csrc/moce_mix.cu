@@ -31,9 +31,13 @@ __global__ void __launch_bounds__(kThreads) mix_nchw_kernel(const T *__restrict_
                                                             const int32_t *__restrict__ pidx,
                                                             const float *__restrict__ a,
                                                             const int32_t *__restrict__ resid,
-                                                            int nU, int EPB, T *__restrict__ y) {
+                                                            int nU, int EPB, T *__restrict__ y,
+                                                            PerExample pe) {
     const int p = blockIdx.x * kThreads + threadIdx.x;
     const int n = blockIdx.z;
+    pidx += (size_t)n * pe.sup_stride;
+    resid += (size_t)n * pe.resid_stride;
+    if (pe.nUa) nU = pe.nUa[n];
     const int e0 = blockIdx.y * EPB, e1 = min(R + 1, e0 + EPB);
     if (p >= HW) return;
     const T *xn = x + (size_t)n * C * HW + p;
@@ -56,7 +60,8 @@ __global__ void __launch_bounds__(kThreads) mix_nchw_kernel(const T *__restrict_
 template <typename T>
 __global__ void __launch_bounds__(kThreads) mix_nhwc_generic_kernel(
     const T *__restrict__ x, int N, int HW, int C, int R, int k, const int32_t *__restrict__ pidx,
-    const float *__restrict__ a, const int32_t *__restrict__ resid, int nU, T *__restrict__ y) {
+    const float *__restrict__ a, const int32_t *__restrict__ resid, int nU, T *__restrict__ y,
+    PerExample pe) {
     const size_t total = (size_t)N * HW * (R + 1);
     for (size_t q = (size_t)blockIdx.x * kThreads + threadIdx.x; q < total;
          q += (size_t)gridDim.x * kThreads) {
@@ -66,12 +71,16 @@ __global__ void __launch_bounds__(kThreads) mix_nhwc_generic_kernel(
         const T *xp = x + np * C;
         float acc = 0.f;
         if (e < R) {
-            const int32_t *ie = pidx + (size_t)e * k;
+            const int32_t *ie = pidx + n * pe.sup_stride + (size_t)e * k;
             const float *ae = a + (n * R + e) * k;
             for (int i = 0; i < k; ++i) acc = fmaf(__ldg(ae + i), load_elem<T>(xp + __ldg(ie + i)), acc);
-        } else if (nU > 0) {
-            for (int j = 0; j < nU; ++j) acc += load_elem<T>(xp + __ldg(resid + j));
-            acc = acc / (float)nU;
+        } else {
+            const int nUn = pe.nUa ? pe.nUa[n] : nU;
+            const int32_t *rn = resid + n * pe.resid_stride;
+            if (nUn > 0) {
+                for (int j = 0; j < nUn; ++j) acc += load_elem<T>(xp + __ldg(rn + j));
+                acc = acc / (float)nUn;
+            }
         }
         y[q] = store_cvt<T>(acc);
     }
@@ -81,23 +90,24 @@ template <int GS>
 __global__ void __launch_bounds__(kThreads) mix_nhwc_bf16_tiled_kernel(
     const uint16_t *__restrict__ x, int HW, int C, int R, int k, const int32_t *__restrict__ pidx,
     const float *__restrict__ a, const int32_t *__restrict__ resid, int nU,
-    uint16_t *__restrict__ y, int tiles, MixGeom geom) {
+    uint16_t *__restrict__ y, int tiles, MixGeom geom, PerExample pe) {
     extern __shared__ __align__(16) unsigned char msm[];
     const int n = blockIdx.x / tiles, t = blockIdx.x - n * tiles;
-    mix_nhwc_bf16_tile<GS>(msm, geom, x, HW, C, R, k, pidx, a + (size_t)n * R * k, resid, nU, y, n,
-                           t);
+    mix_nhwc_bf16_tile<GS>(msm, geom, x, HW, C, R, k, pidx + (size_t)n * pe.sup_stride,
+                           a + (size_t)n * R * k, resid + (size_t)n * pe.resid_stride,
+                           pe.nUa ? pe.nUa[n] : nU, y, n, t);
 }
 
 template <int GS>
 cudaError_t launch_tiled(const uint16_t *x, int N, int HW, int C, int R, int k,
                          const int32_t *pidx, const float *a, const int32_t *resid, int nU,
-                         uint16_t *y, const MixGeom &g, cudaStream_t s) {
+                         uint16_t *y, const MixGeom &g, const PerExample &pe, cudaStream_t s) {
     cudaError_t err = cudaFuncSetAttribute(mix_nhwc_bf16_tiled_kernel<GS>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
     if (err != cudaSuccess) return err;
     const int tiles = (HW + g.TP - 1) / g.TP;
     mix_nhwc_bf16_tiled_kernel<GS><<<(unsigned)((size_t)N * tiles), kThreads, g.smem, s>>>(
-        x, HW, C, R, k, pidx, a, resid, nU, y, tiles, g);
+        x, HW, C, R, k, pidx, a, resid, nU, y, tiles, g, pe);
     return cudaGetLastError();
 }
 
@@ -155,21 +165,23 @@ bool mix_geometry(int C, int R, int k, size_t budget, MixGeom *out) {
 
 cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
                        moce_layout_t lay, const int32_t *pidx, const float *a,
-                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s) {
+                       const int32_t *resid, int nU, void *y, uint32_t *ctrl, cudaStream_t s,
+                       const PerExample &pe) {
     if (N == 0 || HW == 0) return cudaSuccess;
+    const bool shared = pe.sup_stride == 0 && pe.resid_stride == 0 && pe.nUa == nullptr;
     if (lay == MOCE_NCHW) {
         const int EPB = 8;
         const dim3 grid((HW + kThreads - 1) / kThreads, (R + 1 + EPB - 1) / EPB, N);
         if (dt == MOCE_BF16)
             mix_nchw_kernel<uint16_t><<<grid, kThreads, 0, s>>>((const uint16_t *)x, HW, C, R, k,
                                                                  pidx, a, resid, nU, EPB,
-                                                                 (uint16_t *)y);
+                                                                 (uint16_t *)y, pe);
         else
             mix_nchw_kernel<float><<<grid, kThreads, 0, s>>>((const float *)x, HW, C, R, k, pidx, a,
-                                                              resid, nU, EPB, (float *)y);
+                                                              resid, nU, EPB, (float *)y, pe);
         return cudaGetLastError();
     }
-    if (dt == MOCE_BF16 && C % 8 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
+    if (shared && dt == MOCE_BF16 && C % 8 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
         (reinterpret_cast<uintptr_t>(pidx) & 15u) == 0 &&
         (reinterpret_cast<uintptr_t>(a) & 15u) == 0 && mix_wide_supported(HW, C, R, k, nU))
         return launch_mix_wide((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU,
@@ -180,10 +192,10 @@ cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_d
                        mix_geometry(C, R, k, kMixSmemBudget, &g);
     if (tiled) {
         switch (g.GS) {
-        case 16: return launch_tiled<16>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, s);
-        case 8: return launch_tiled<8>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, s);
-        case 4: return launch_tiled<4>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, s);
-        default: return launch_tiled<2>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, s);
+        case 16: return launch_tiled<16>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, pe, s);
+        case 8: return launch_tiled<8>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, pe, s);
+        case 4: return launch_tiled<4>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, pe, s);
+        default: return launch_tiled<2>((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, g, pe, s);
         }
     }
     const size_t total = (size_t)N * HW * (R + 1);
@@ -191,10 +203,10 @@ cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_d
     if (blocks > 65535u * 16u) blocks = 65535u * 16u;
     if (dt == MOCE_BF16)
         mix_nhwc_generic_kernel<uint16_t><<<(unsigned)blocks, kThreads, 0, s>>>(
-            (const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y);
+            (const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU, (uint16_t *)y, pe);
     else
         mix_nhwc_generic_kernel<float><<<(unsigned)blocks, kThreads, 0, s>>>(
-            (const float *)x, N, HW, C, R, k, pidx, a, resid, nU, (float *)y);
+            (const float *)x, N, HW, C, R, k, pidx, a, resid, nU, (float *)y, pe);
     return cudaGetLastError();
 }
 

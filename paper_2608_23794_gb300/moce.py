@@ -74,6 +74,13 @@ def library():
             "moce_topk_supports": ([P, I, I, I, P, P, P, S, P], I),
             "moce_coverage_loss": ([P, I, I, F, P, P, P, P, S, P], I),
             "moce_backward_workspace_bytes": ([I, I, I, I, I, I], S),
+            "moce_mix": ([P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, S, P], I),
+            "moce_dynamic_workspace_bytes": ([I, I, I, I, I, I, I], S),
+            "moce_dynamic_supports": ([P, I, I, I, I, I, P, P, P, P, P, P, P, P, P, P, S, P], I),
+            "moce_forward_supports": ([P, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P, F, F, P,
+                                       P, S, P], I),
+            "moce_forward_dynamic": ([P, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P, P, F, F,
+                                      P, P, P, P, P, S, P], I),
             "moce_backward": ([P, P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, P, F, F,
                                P, P, P, P, P, P, P, S, P], I),
         }
@@ -383,6 +390,131 @@ def moce_backward(x: torch.Tensor, dy: torch.Tensor, layout: str, packed: Packed
                                    _ptr(g.dW1), _ptr(g.db1), _ptr(g.dw2), _ptr(g.db2), _ptr(ws),
                                    ws.numel(), _stream(stream)), "moce_backward")
     return g
+
+
+def moce_mix(x: torch.Tensor, layout: str, sup_idx: torch.Tensor, mix_w: torch.Tensor,
+             resid_idx: torch.Tensor, n_resid, ws: Workspace, y: torch.Tensor | None = None,
+             stream=None) -> torch.Tensor:
+    """Eq. (expert) and Eq. (res) from weights mix_w [N, C_out, k].
+
+    Shared supports: sup_idx [C_out, k], resid_idx [C_in], n_resid an int. Per-example
+    supports: sup_idx [N, C_out, k], resid_idx [N, C_in], n_resid an int32 CUDA tensor [N].
+    """
+    N, H, W, C = _dims(x, layout)
+    R, k = sup_idx.shape[-2], sup_idx.shape[-1]
+    if y is None:
+        shape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+        y = torch.empty(shape, dtype=x.dtype, device=x.device)
+    per = isinstance(n_resid, torch.Tensor)
+    _check(library().moce_mix(_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout],
+                              _ptr(sup_idx), _ptr(mix_w), _ptr(resid_idx),
+                              0 if per else int(n_resid), _ptr(n_resid) if per else None, _ptr(y),
+                              _ptr(ws.buffer), ws.nbytes, _stream(stream)), "moce_mix")
+    return y
+
+
+@dataclass
+class DynamicRouter:
+    """Parameters of Eq. (dynamic): the static routing matrix and the rank-d router."""
+    logits: torch.Tensor   # float32 [C_out, C_in]
+    Wh: torch.Tensor       # float32 [d, C_in]
+    bh: torch.Tensor       # float32 [d]
+    V: torch.Tensor        # float32 [C_in, d], row c = v_c
+    Q: torch.Tensor        # float32 [C_out, d], row e = q_e
+
+    @property
+    def d(self) -> int:
+        return self.Wh.shape[0]
+
+
+@dataclass
+class DynamicSupports:
+    sup_idx: torch.Tensor     # int32 [N, C_out, k], deployment order per example
+    sup_logits: torch.Tensor  # float32 [N, C_out, k]: the selected L_e(X) values
+    resid_idx: torch.Tensor   # int32 [N, C_in]: row n starts with U(X) ascending
+    n_resid: torch.Tensor     # int32 [N]
+
+
+def moce_dynamic_workspace_bytes(N, H, W, C_in, C_out, k, d) -> int:
+    return int(library().moce_dynamic_workspace_bytes(N, H, W, C_in, C_out, k, d))
+
+
+def _dyn_ws(N, H, W, C, R, k, d, device):
+    nbytes = moce_dynamic_workspace_bytes(N, H, W, C, R, k, d)
+    if nbytes == 0:
+        raise MoceError(MOCE_ERR_UNSUPPORTED, "moce_dynamic_workspace_bytes")
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def _empty_supports(N, R, k, C, device) -> DynamicSupports:
+    return DynamicSupports(torch.empty((N, R, k), dtype=torch.int32, device=device),
+                           torch.empty((N, R, k), dtype=torch.float32, device=device),
+                           torch.empty((N, C), dtype=torch.int32, device=device),
+                           torch.empty(N, dtype=torch.int32, device=device))
+
+
+def moce_dynamic_supports(z: torch.Tensor, router: DynamicRouter, k: int,
+                          ws: torch.Tensor | None = None, out: DynamicSupports | None = None,
+                          stream=None) -> DynamicSupports:
+    """Per-example supports of Eq. (dynamic) from pooled descriptors z [N, C_in]."""
+    N, C = z.shape
+    R, d = router.logits.shape[0], router.d
+    sup = out or _empty_supports(N, R, k, C, z.device)
+    if ws is None:
+        ws = _dyn_ws(N, 1, 1, C, R, k, d, z.device)
+    _check(library().moce_dynamic_supports(_ptr(z), N, C, R, k, d, _ptr(router.logits),
+                                           _ptr(router.Wh), _ptr(router.bh), _ptr(router.V),
+                                           _ptr(router.Q), _ptr(sup.sup_idx), _ptr(sup.sup_logits),
+                                           _ptr(sup.resid_idx), _ptr(sup.n_resid), _ptr(ws),
+                                           ws.numel(), _stream(stream)), "moce_dynamic_supports")
+    return sup
+
+
+def moce_forward_supports(x: torch.Tensor, layout: str, sup: DynamicSupports, W1, b1, w2, b2,
+                          tau_min: float, tau_max: float, ws: Workspace | None = None,
+                          y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """The layer with given per-example supports (pool, gate, mix)."""
+    N, H, W, C = _dims(x, layout)
+    R, k = sup.sup_idx.shape[1], sup.sup_idx.shape[2]
+    if y is None:
+        shape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+        y = torch.empty(shape, dtype=x.dtype, device=x.device)
+    if ws is None:
+        ws = Workspace(N, H, W, C, R, k, device=x.device)
+    _check(library().moce_forward_supports(_ptr(x), N, H, W, C, R, k, _dtype(x), _LAYOUTS[layout],
+                                           _ptr(sup.sup_idx), _ptr(sup.sup_logits),
+                                           _ptr(sup.resid_idx), _ptr(sup.n_resid), _ptr(W1),
+                                           _ptr(b1), _ptr(w2), _ptr(b2), float(tau_min),
+                                           float(tau_max), _ptr(y), _ptr(ws.buffer), ws.nbytes,
+                                           _stream(stream)), "moce_forward_supports")
+    return y
+
+
+def moce_forward_dynamic(x: torch.Tensor, layout: str, router: DynamicRouter, k: int, W1, b1, w2,
+                         b2, tau_min: float, tau_max: float, ws: torch.Tensor | None = None,
+                         y: torch.Tensor | None = None, supports: DynamicSupports | None = None,
+                         stream=None) -> torch.Tensor:
+    """The input-conditioned support variant (Eq. dynamic), inference path.
+
+    ``supports`` (optional) receives the per-example supports and |U(X)|; its resid_idx is
+    not written (U(X) stays in the workspace).
+    """
+    N, H, W, C = _dims(x, layout)
+    R, d = router.logits.shape[0], router.d
+    if y is None:
+        shape = (N, H, W, R + 1) if layout == "nhwc" else (N, R + 1, H, W)
+        y = torch.empty(shape, dtype=x.dtype, device=x.device)
+    if ws is None:
+        ws = _dyn_ws(N, H, W, C, R, k, d, x.device)
+    _check(library().moce_forward_dynamic(
+        _ptr(x), N, H, W, C, R, k, d, _dtype(x), _LAYOUTS[layout], _ptr(router.logits),
+        _ptr(router.Wh), _ptr(router.bh), _ptr(router.V), _ptr(router.Q), _ptr(W1), _ptr(b1),
+        _ptr(w2), _ptr(b2), float(tau_min), float(tau_max), _ptr(y),
+        _ptr(supports.sup_idx) if supports else None,
+        _ptr(supports.sup_logits) if supports else None,
+        _ptr(supports.n_resid) if supports else None, _ptr(ws), ws.numel(), _stream(stream)),
+        "moce_forward_dynamic")
+    return y
 
 
 def moce_noalloc_check_device_error(stream=None):

@@ -208,6 +208,45 @@ def make_dy(cfg: LayerConfig, seed: int = 0):
     return a, bits
 
 
+def make_dynamic_x(cfg: LayerConfig, seed: int = 0, mean_std: float = 0.5,
+                   grid: float | None = None):
+    """Activations for the input-conditioned variant: act(N(mu[n, c], 1)) with per-example
+    channel means mu ~ N(0, mean_std^2), so that the pooled descriptors (the router's input)
+    differ between examples as real feature maps do. With `grid`, values are rounded to
+    multiples of it (1/16: every partial sum of a pool is then exact in fp32). Returns
+    (float32 values, bf16 bits or None) in cfg.layout."""
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0xD1]))
+    mu = (rng.standard_normal((cfg.N, 1, 1, cfg.C_in)) * mean_std).astype(np.float32)
+    a = rng.standard_normal((cfg.N, cfg.H, cfg.W, cfg.C_in), dtype=np.float32) + mu
+    if cfg.activation == "relu":
+        np.maximum(a, np.float32(0.0), out=a)
+    else:
+        a = _gelu(a)
+    if grid is not None:
+        a = (np.round(a / np.float32(grid)) * np.float32(grid)).astype(np.float32)
+    if cfg.layout == "nchw":
+        a = np.ascontiguousarray(a.transpose(0, 3, 1, 2))
+    bits = None
+    if cfg.dtype == "bf16":
+        bits = bf16_bits(a)
+        a = bf16_to_f32(bits)
+    return a, bits
+
+
+def make_router(cfg: LayerConfig, d: int, seed: int = 0):
+    """Parameters of the rank-d router of Eq. (dynamic): the static routing matrix L ~ N(0, 1)
+    [C_out, C_in], W_h ~ N(0, 1/C_in) [d, C_in], b_h ~ N(0, 0.01) [d], v_c ~ N(0, 1/d) [C_in, d],
+    q_e ~ N(0, 4) [C_out, d] (so the offset is of the order of the logits' spread)."""
+    rng = np.random.default_rng(np.random.SeedSequence([seed, 0xD2]))
+    R, C = cfg.C_out, cfg.C_in
+    f = np.float32
+    return {"L": rng.standard_normal((R, C), dtype=f),
+            "Wh": (rng.standard_normal((d, C), dtype=f) / f(np.sqrt(C))).astype(f),
+            "bh": (rng.standard_normal(d, dtype=f) * f(0.1)).astype(f),
+            "V": (rng.standard_normal((C, d), dtype=f) / f(np.sqrt(d))).astype(f),
+            "Q": (rng.standard_normal((R, d), dtype=f) * f(2.0)).astype(f)}
+
+
 def x_to_layout(x: np.ndarray, src: str, dst: str) -> np.ndarray:
     if src == dst:
         return x

@@ -164,6 +164,45 @@ def test_backward_rejects_bad_arguments_on_host(lib):
     assert call(C=6000, nU=0) == 3                # valid, no kernel for it
 
 
+def test_dynamic_rejects_bad_arguments_on_host(lib):
+    P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    wb = lib.moce_dynamic_workspace_bytes
+    wb.argtypes, wb.restype = [I] * 7, S
+    assert wb(2, 4, 4, 64, 8, 4, 16) > 0
+    assert wb(2, 4, 4, 64, 8, 4, 0) == 0          # d < 1
+    assert wb(2, 4, 4, 20000, 8, 4, 16) == 0      # C_in beyond the shared-memory TopK
+    # the routing buffers do not depend on H, W: a larger H W only adds the forward part
+    assert wb(2, 64, 64, 64, 8, 4, 16) > wb(2, 4, 4, 64, 8, 4, 16)
+    f = lib.moce_forward_dynamic
+    f.argtypes = [P, I, I, I, I, I, I, I, I, I, P, P, P, P, P, P, P, P, P, F, F, P, P, P, P, P, S, P]
+    f.restype = I
+    fake = ctypes.c_void_p(0x1000)
+    good = dict(N=2, C=64, R=8, k=4, d=16, dt=1, lay=0, tmin=0.2, tmax=6.0, ws=fake, wsb=1 << 40)
+
+    def call(**kw):
+        a = {**good, **kw}
+        return f(fake, a["N"], 4, 4, a["C"], a["R"], a["k"], a["d"], a["dt"], a["lay"], fake, fake,
+                 fake, fake, fake, fake, fake, fake, fake, a["tmin"], a["tmax"], fake, None, None,
+                 None, a["ws"], a["wsb"], None)
+
+    assert call(d=0) == 1
+    assert call(k=65) == 1
+    assert call(dt=3) == 1
+    assert call(tmin=0.0) == 1
+    assert call(ws=None) == 1
+    assert call(wsb=64) == 1
+    assert call(ws=ctypes.c_void_p(0x1080)) == 1     # not 256-byte aligned
+    assert call(C=20000, k=4) == 3                    # valid, TopK row does not fit
+    assert call(N=0) == 0
+    m = lib.moce_mix
+    m.argtypes = [P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, S, P]
+    m.restype = I
+    assert m(fake, 2, 4, 4, 64, 8, 4, 1, 0, fake, fake, fake, 65, None, fake, fake, 1 << 40,
+             None) == 1                               # |U| > C_in
+    assert m(fake, 2, 4, 4, 64, 8, 4, 1, 0, fake, fake, None, 0, fake, fake, fake, 1 << 40,
+             None) == 1                               # per-example U without its rows
+
+
 def test_pack_rejects_bad_arguments_on_host(lib):
     f = lib.moce_pack_supports
     P, I = ctypes.c_void_p, ctypes.c_int
