@@ -54,10 +54,13 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto",
                     help="kernel path of the forward (auto, stream, steps)")
-    ap.add_argument("--op", choices=["forward", "backward", "train"], default="forward",
+    ap.add_argument("--d", type=int, default=32,
+                    help="router rank of the input-conditioned variant (--op dynamic)")
+    ap.add_argument("--op", choices=["forward", "backward", "train", "dynamic"], default="forward",
                     help="forward: the layer forward (the benchmark); backward: the layer's "
                          "gradients for an upstream gradient; train: TopK over the full "
-                         "routing matrix and the coverage loss with its gradient")
+                         "routing matrix and the coverage loss with its gradient; dynamic: "
+                         "static against input-conditioned supports (Eq. dynamic)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline leg")
     return ap.parse_args()
@@ -700,6 +703,105 @@ def run_backward(args, cfg):
     print(json.dumps(line), flush=True)
 
 
+def run_dynamic(args, cfg):
+    """Static supports against the input-conditioned variant of Eq. (dynamic) on the same layer
+    and inputs (Sec. 5 compares the two): device µs per call of the whole layer for each, and of
+    the paper's "routing-and-gather" path, i.e. the static indexed mix against the dynamic
+    router (hidden layer, rank-d logits, per-example TopK, U(X)) plus the per-example mix. The
+    mix kernels fuse the gather with the aggregation, so both sides include the aggregation."""
+    import numpy as np
+    import torch
+
+    from paper_2608_23794_gb300 import build as moce_build
+    from paper_2608_23794_gb300 import moce, synth
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    moce_build.build()
+    d = args.d
+    lay = synth.make_layer(cfg, seed=SEED)
+    xv, xb = synth.make_dynamic_x(cfg, seed=SEED)
+    rt = synth.make_router(cfg, d, seed=SEED)
+    cu = lambda a, dt=torch.float32: torch.from_numpy(np.ascontiguousarray(a)).to(dev, dt)
+    x = (torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16) if xb is not None
+         else torch.from_numpy(xv))
+    router = moce.DynamicRouter(cu(rt["L"]), cu(rt["Wh"]), cu(rt["bh"]), cu(rt["V"]), cu(rt["Q"]))
+    gate = (cu(lay.W1), cu(lay.b1), cu(lay.w2), cu(lay.b2))
+    N, R, k, C = cfg.N, cfg.C_out, cfg.k, cfg.C_in
+    # the static layer selects TopK of the same routing matrix, packed once
+    idx_t, lg_t = moce.moce_topk_supports(router.logits, k)
+    packed = moce.moce_pack_supports(idx_t, lg_t, C)
+    s_el = 2 if cfg.dtype == "bf16" else 4
+    x_bytes = N * cfg.H * cfg.W * C * s_el
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 132 * 2**20
+    n_rot = max(2, int(np.ceil(3 * l2 / x_bytes)) + 1)
+    xs = [x.to(dev) for _ in range(n_rot)]
+    shape_y = (N, cfg.H, cfg.W, R + 1) if cfg.layout == "nhwc" else (N, R + 1, cfg.H, cfg.W)
+    ys = [torch.empty(shape_y, dtype=xs[0].dtype, device=dev) for _ in range(n_rot)]
+    ws = moce.Workspace(N, cfg.H, cfg.W, C, R, k, device=dev)
+    dws = torch.empty(moce.moce_dynamic_workspace_bytes(N, cfg.H, cfg.W, C, R, k, d),
+                      dtype=torch.uint8, device=dev)
+    sup = moce._empty_supports(N, R, k, C, dev)
+    z = moce.moce_pool(xs[0], cfg.layout)
+    _, a_static = moce.moce_gate(z, packed, *gate, cfg.tau_min, cfg.tau_max)
+    a_dyn = torch.empty((N, R, k), dtype=torch.float32, device=dev)
+    moce.moce_dynamic_supports(z, router, k, ws=dws, out=sup)
+    resid_static = packed.resid_idx
+    K = max(3, min(args.steps, 500))
+
+    def timed(fn):
+        for i in range(max(3, args.warmup)):
+            fn(i)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(K):
+            fn(i)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / K
+
+    sampler = ClockSampler(gpu_uuid(torch, dev))
+    sampler.start()
+    time.sleep(0.3)
+    t_static = timed(lambda i: moce.moce_forward(xs[i % n_rot], cfg.layout, packed, *gate,
+                                                 cfg.tau_min, cfg.tau_max, ws=ws,
+                                                 y=ys[i % n_rot]))
+    t_dyn = timed(lambda i: moce.moce_forward_dynamic(xs[i % n_rot], cfg.layout, router, k, *gate,
+                                                      cfg.tau_min, cfg.tau_max, ws=dws,
+                                                      y=ys[i % n_rot]))
+    t_mix_static = timed(lambda i: moce.moce_mix(xs[i % n_rot], cfg.layout,
+                                                 packed.packed_idx.view(R, k), a_static,
+                                                 resid_static, packed.n_resid, ws,
+                                                 y=ys[i % n_rot]))
+    t_route = timed(lambda i: moce.moce_dynamic_supports(z, router, k, ws=dws, out=sup))
+    t_mix_dyn = timed(lambda i: moce.moce_mix(xs[i % n_rot], cfg.layout, sup.sup_idx, a_dyn,
+                                              sup.resid_idx, sup.n_resid, ws, y=ys[i % n_rot]))
+    clocks = sampler.stop()
+    rg_static = t_mix_static
+    rg_dyn = t_route + t_mix_dyn
+    line = {"metric": "MoCE static vs input-conditioned supports (Eq. dynamic): µs per layer and "
+                      "routing-and-gather ratio",
+            "value": rg_dyn / rg_static, "unit": "x (dynamic / static routing-and-gather time)",
+            "n_gpus": 1, "steps": K, "warmup": args.warmup, "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": DATA[cfg.activation] +
+            "; per-example channel means N(0, 0.25) so the router sees different descriptors",
+            "config": {"workload": cfg.name, "N": N, "H": cfg.H, "W": cfg.W, "C_in": C,
+                       "C_out": R, "k": k, "d": d, "storage_dtype": cfg.dtype,
+                       "layout": cfg.layout, "op": "dynamic",
+                       "l2": f"{n_rot} rotating input copies (> L2)"},
+            "static": {"layer_us": t_static, "mix_us": t_mix_static},
+            "dynamic": {"layer_us": t_dyn, "route_us": t_route, "mix_us": t_mix_dyn,
+                        "route_note": "router hidden layer, rank-d logits of every (expert, "
+                                      "channel), per-example TopK, U(X)"},
+            "ratio_layer": t_dyn / t_static,
+            "ratio_routing_and_gather": rg_dyn / rg_static,
+            "paper_ratio_routing_and_gather": 13.5 / 1.9,
+            "clocks": clocks, "gpu_launches": None}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     from paper_2608_23794_gb300 import synth
@@ -709,6 +811,9 @@ def main():
         return
     if args.op == "backward":
         run_backward(args, cfg)
+        return
+    if args.op == "dynamic":
+        run_dynamic(args, cfg)
         return
     if args.impl == "ours" and (cfg.dtype, cfg.layout) != ("bf16", "nhwc"):
         raise SystemExit(f"bench.py times bf16 NHWC layers; {cfg.name} is {cfg.dtype} {cfg.layout}")

@@ -250,7 +250,7 @@ moce_status_t moce_topk_supports(const float *logits, int C_in, int C_out, int k
     if (!logits || !packed_idx || !packed_logits || !ws) return MOCE_ERR_INVALID_VALUE;
     if (ws_bytes < train_ws_bytes(C_out, C_in) || (reinterpret_cast<uintptr_t>(ws) & 255u))
         return MOCE_ERR_INVALID_VALUE;
-    if ((size_t)topk_padded(C_in) * 8 > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
+    if (topk_smem_bytes(C_in, k) > 227 * 1024) return MOCE_ERR_UNSUPPORTED;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     uint32_t *err_word = static_cast<uint32_t *>(ws);
     cudaError_t err = cudaMemsetAsync(err_word, 0, 4, s);
@@ -310,7 +310,7 @@ static bool dyn_shape_ok(int N, int H, int W, int C_in, int C_out, int k, int d)
 }
 
 size_t moce_dynamic_workspace_bytes(int N, int H, int W, int C_in, int C_out, int k, int d) {
-    if (!dyn_shape_ok(N, H, W, C_in, C_out, k, d) || !dynamic_supported(C_in)) return 0;
+    if (!dyn_shape_ok(N, H, W, C_in, C_out, k, d) || !dynamic_supported(C_in, k)) return 0;
     return dyn_layout(N, H * W, C_in, C_out, k, d).total;
 }
 
@@ -320,7 +320,7 @@ moce_status_t moce_dynamic_supports(const float *z, int N, int C_in, int C_out, 
                                     float *sup_logits, int32_t *resid_idx, int32_t *n_resid,
                                     void *ws, size_t ws_bytes, moce_stream_t stream) {
     if (!dyn_shape_ok(N, 1, 1, C_in, C_out, k, d)) return MOCE_ERR_INVALID_VALUE;
-    if (!dynamic_supported(C_in)) return MOCE_ERR_UNSUPPORTED;
+    if (!dynamic_supported(C_in, k)) return MOCE_ERR_UNSUPPORTED;
     if (N == 0) return MOCE_OK;
     if (!z || !logits || !Wh || !bh || !V || !Q || !sup_idx || !sup_logits || !resid_idx ||
         !n_resid || !ws)
@@ -395,7 +395,7 @@ moce_status_t moce_forward_dynamic(const void *x, int N, int H, int W, int C_in,
     if (!dyn_shape_ok(N, H, W, C_in, C_out, k, d) || !dtype_ok(dtype) || !layout_ok(layout) ||
         !tau_ok(tau_min, tau_max))
         return MOCE_ERR_INVALID_VALUE;
-    if (!dynamic_supported(C_in)) return MOCE_ERR_UNSUPPORTED;
+    if (!dynamic_supported(C_in, k)) return MOCE_ERR_UNSUPPORTED;
     const int HW = H * W;
     if (N == 0 || HW == 0) return MOCE_OK;
     if (!x || !logits || !Wh || !bh || !V || !Q || !W1 || !b1 || !w2 || !b2 || !y || !ws)

@@ -152,8 +152,8 @@ DynLayout dyn_layout(int N, int HW, int C, int R, int k, int d) {
     return D;
 }
 
-bool dynamic_supported(int C) {
-    return (size_t)topk_padded(C) * 8 <= 227 * 1024 && (size_t)((C + 31) / 32) * 4 <= 64 * 1024;
+bool dynamic_supported(int C, int k) {
+    return topk_smem_bytes(C, k) <= 227 * 1024 && (size_t)((C + 31) / 32) * 4 <= 64 * 1024;
 }
 
 cudaError_t launch_dynamic_supports(const float *z, int N, int C, int R, int k, int d,

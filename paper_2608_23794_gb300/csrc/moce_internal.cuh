@@ -114,6 +114,14 @@ struct MixGeom {
 
 bool mix_geometry(int C, int R, int k, size_t smem_budget, MixGeom *g);
 
+// Per-example supports of the mixing kernels: example n reads its supports
+// at pidx + n sup_stride, its U at resid + n resid_stride and |U| at nUa[n]
+// (a device array; when nUa is null every example has the scalar nU).
+struct PerExample {
+    size_t sup_stride = 0, resid_stride = 0;
+    const int32_t *nUa = nullptr;
+};
+
 // ---------------------------------------------------------------- launchers (host)
 cudaError_t launch_pack(int C, int R, int k, const int32_t *idx, const float *lg, int32_t *pidx,
                         float *plog, int32_t *resid, uint32_t *ws_words, cudaStream_t s);
@@ -128,14 +136,6 @@ cudaError_t launch_gate(const float *z, int N, int C, int R, int k, const int32_
                         const float *b2, float tmin, float tmax, float *tau, float *a,
                         cudaStream_t s, size_t sup_stride = 0);
 
-// Per-example supports of the mixing kernels: example n reads its supports
-// at pidx + n sup_stride, its U at resid + n resid_stride and |U| at nUa[n]
-// (a device array; when nUa is null every example has the scalar nU).
-struct PerExample {
-    size_t sup_stride = 0, resid_stride = 0;
-    const int32_t *nUa = nullptr;
-};
-
 // ctrl: the workspace control words (bounded waits report MOCE_ERR_TIMEOUT there).
 cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_dtype_t dt,
                        moce_layout_t lay, const int32_t *pidx, const float *a,
@@ -147,11 +147,13 @@ cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_d
 bool mix_wide_supported(int HW, int C, int R, int k, int nU);
 cudaError_t launch_mix_wide(const uint16_t *x, int N, int HW, int C, int R, int k,
                             const int32_t *pidx, const float *a, const int32_t *resid, int nU,
-                            uint16_t *y, uint32_t *ctrl, cudaStream_t s);
+                            uint16_t *y, uint32_t *ctrl, cudaStream_t s, const PerExample &pe);
 
 // Support maintenance (moce_train.cu): TopK over full routing rows and the
 // coverage regularizer.
-int topk_padded(int C);
+// Shared memory of one TopK row (the k selected pairs padded to a power of
+// two, and the row's order keys).
+size_t topk_smem_bytes(int C, int k);
 size_t train_ws_bytes(int R, int C);
 cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float *lg,
                         uint32_t *err, cudaStream_t s);
@@ -179,7 +181,7 @@ struct DynLayout {
     size_t total = 0;
 };
 DynLayout dyn_layout(int N, int HW, int C, int R, int k, int d);
-bool dynamic_supported(int C);
+bool dynamic_supported(int C, int k);
 // From pooled descriptors z [N][C]: h [N][d], the logits Ld [N][R][C], the
 // per-example supports sidx / slog [N][R][k] (deployment order), U(X) in
 // resid [N][C] (ascending) and |U(X)| in nU [N]. err: TopK's non-finite flag.

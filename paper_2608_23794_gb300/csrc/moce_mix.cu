@@ -4,7 +4,7 @@
 // The weights a[n,e,i] come from the gate stage. fp32 accumulation, output
 // rounded to the input dtype (bf16: round to nearest even).
 //
-// NHWC bf16 with C % 8 == 0, k % 8 == 0 and aligned tables goes to
+// NHWC bf16 with C >= 512, C % 8 == 0, k % 8 == 0 and aligned tables goes to
 // mix_wide_kernel (moce_mix_wide.cu); here:
 //  * mix_nchw_kernel: one thread per position, channel planes are contiguous
 //    so a warp's gathered loads are coalesced; any dtype.
@@ -181,11 +181,14 @@ cudaError_t launch_mix(const void *x, int N, int HW, int C, int R, int k, moce_d
                                                               resid, nU, EPB, (float *)y, pe);
         return cudaGetLastError();
     }
-    if (shared && dt == MOCE_BF16 && C % 8 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
+    // the wide kernel pays off from 512 channels (at 256 the tiled kernel is faster)
+    if (C >= 512 && dt == MOCE_BF16 && C % 8 == 0 &&
+        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&
         (reinterpret_cast<uintptr_t>(pidx) & 15u) == 0 &&
-        (reinterpret_cast<uintptr_t>(a) & 15u) == 0 && mix_wide_supported(HW, C, R, k, nU))
+        (reinterpret_cast<uintptr_t>(a) & 15u) == 0 &&
+        mix_wide_supported(HW, C, R, k, shared ? nU : C))
         return launch_mix_wide((const uint16_t *)x, N, HW, C, R, k, pidx, a, resid, nU,
-                               (uint16_t *)y, ctrl, s);
+                               (uint16_t *)y, ctrl, s, pe);
     MixGeom g;
     const bool tiled = dt == MOCE_BF16 && C % 8 == 0 &&
                        (reinterpret_cast<uintptr_t>(x) & 15u) == 0 &&

@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kWideThreads, 1) mix_wide_kernel(
     const uint16_t *__restrict__ x, int HW, int C, int R, int k,
     const int32_t *__restrict__ pidx, const float *__restrict__ a,
     const int32_t *__restrict__ resid, int nU, uint16_t *__restrict__ y, uint32_t *ctrl,
-    WideGeom g) {
+    WideGeom g, PerExample pe) {
     constexpr int TP = 8 * GS, RB = 16 * GS, FM = GS - 1;
     extern __shared__ __align__(128) unsigned char wsm[];
     unsigned char *xs = wsm;
@@ -154,6 +154,9 @@ __global__ void __launch_bounds__(kWideThreads, 1) mix_wide_kernel(
     const int p0 = t * TP, np = min(TP, HW - p0);
     const int E = R + 1;
     const float *an = a + (size_t)n * R * k;
+    pidx += (size_t)n * pe.sup_stride;  // per-example supports (0: shared)
+    resid += (size_t)n * pe.resid_stride;
+    if (pe.nUa) nU = pe.nUa[n];
     const int nch = (R + g.EB - 1) / g.EB;
     // table chunk j: the support indices, then the weights, of experts
     // j EB .. j EB + EB - 1 (each a contiguous run of rows in global memory)
@@ -351,12 +354,13 @@ bool wide_geometry(int HW, int C, int R, int k, int nU, WideGeom *out) {
 template <int GS>
 cudaError_t launch_wide_gs(const uint16_t *x, int N, int HW, int C, int R, int k,
                            const int32_t *pidx, const float *a, const int32_t *resid, int nU,
-                           uint16_t *y, uint32_t *ctrl, const WideGeom &g, cudaStream_t s) {
+                           uint16_t *y, uint32_t *ctrl, const WideGeom &g, const PerExample &pe,
+                           cudaStream_t s) {
     cudaError_t err = cudaFuncSetAttribute(mix_wide_kernel<GS>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
     if (err != cudaSuccess) return err;
     mix_wide_kernel<GS><<<(unsigned)((size_t)N * g.tiles), kWideThreads, g.smem, s>>>(
-        x, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g);
+        x, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, pe);
     return cudaGetLastError();
 }
 
@@ -369,17 +373,18 @@ bool mix_wide_supported(int HW, int C, int R, int k, int nU) {
 
 cudaError_t launch_mix_wide(const uint16_t *x, int N, int HW, int C, int R, int k,
                             const int32_t *pidx, const float *a, const int32_t *resid, int nU,
-                            uint16_t *y, uint32_t *ctrl, cudaStream_t s) {
+                            uint16_t *y, uint32_t *ctrl, cudaStream_t s, const PerExample &pe) {
     WideGeom g;
-    if (C % 8 != 0 || !wide_geometry(HW, C, R, k, nU, &g)) return cudaErrorNotSupported;
+    // per-example U: room for the largest |U(X)| = C
+    if (C % 8 != 0 || !wide_geometry(HW, C, R, k, pe.nUa ? C : nU, &g)) return cudaErrorNotSupported;
     // the bulk copies read 16-byte aligned rows of the tables
     if ((reinterpret_cast<uintptr_t>(pidx) & 15u) || (reinterpret_cast<uintptr_t>(a) & 15u))
         return cudaErrorNotSupported;
     if ((size_t)N * g.tiles > 0x7fffffffu) return cudaErrorNotSupported;
     switch (g.GS) {
-    case 8: return launch_wide_gs<8>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, s);
-    case 4: return launch_wide_gs<4>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, s);
-    default: return launch_wide_gs<2>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, s);
+    case 8: return launch_wide_gs<8>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, pe, s);
+    case 4: return launch_wide_gs<4>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, pe, s);
+    default: return launch_wide_gs<2>(x, N, HW, C, R, k, pidx, a, resid, nU, y, ctrl, g, pe, s);
     }
 }
 

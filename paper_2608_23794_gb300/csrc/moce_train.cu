@@ -1,12 +1,13 @@
 // Support maintenance on the full routing matrix L [R][C] (training side):
 //
-//   topk_rows_kernel      Eq. (support), Sec. 3.2: S_e = TopK(L_e, k), written in
+//   topk_select_kernel    Eq. (support), Sec. 3.2: S_e = TopK(L_e, k), written in
 //                         deployment order (descending logit, equal logits by
 //                         ascending channel; -0.0 equals +0.0), so the result
-//                         is already packed. One CTA per expert row: the row's
-//                         C (key, channel) pairs are sorted in shared memory by
-//                         a bitonic network on 64-bit keys whose high word
-//                         orders the logit and whose low word is the channel.
+//                         is already packed. One CTA per row: a radix select of
+//                         the k-th order key (the key's high word orders the
+//                         logit), an ordered compaction of the k selected
+//                         (key, channel) pairs, then a bitonic sort of only
+//                         those, as 64-bit keys whose low word is the channel.
 //   coverage kernels      Sec. 3.4: p_{e,c} = softmax(L_e)_c over all C channels,
 //                         u_c = (1/R) sum_e p_{e,c}, ubar = (1/C) sum_c u_c,
 //                         L_cov = sum_c (u_c - ubar)^2 / (ubar^2 + eps), and
@@ -69,45 +70,115 @@ __device__ double block_sum_d(double v, double *red) {
     return s;
 }
 
-// One expert row: CP = C rounded up to a power of two keys in shared memory.
-__global__ void __launch_bounds__(kTrainThreads) topk_rows_kernel(const float *__restrict__ L,
-                                                                   int C, int CP, int k,
+// One row per CTA (256 threads): the row's C order keys in shared memory;
+// four 8-bit radix passes find T, the k-th smallest key, and how many of the
+// keys equal to T are taken (the lowest channels first, as the tie rule
+// orders them); an ordered compaction (ballots, in channel order) collects
+// the k selected (key, channel) pairs; a bitonic sort of those KP = k rounded
+// up to a power of two pairs gives deployment order.
+constexpr int kSelThreads = 256;
+__global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float *__restrict__ L,
+                                                                   int C, int k, int KP,
                                                                    int32_t *__restrict__ idx_out,
                                                                    float *__restrict__ lg_out,
                                                                    uint32_t *err) {
-    extern __shared__ unsigned long long keys[];
-    const int e = blockIdx.x;
-    const float *Le = L + (size_t)e * C;
-    for (int c = threadIdx.x; c < CP; c += kTrainThreads) {
-        unsigned long long key = ~0ull;
-        if (c < C) {
-            const float v = Le[c];
-            if (!isfinite(v)) atomicOr(err, kTopkBadLogit);
-            key = ((unsigned long long)desc_key(v) << 32) | (uint32_t)c;
-        }
-        keys[c] = key;
+    extern __shared__ __align__(8) unsigned char ksm[];
+    unsigned long long *sel = reinterpret_cast<unsigned long long *>(ksm);  // [KP]
+    uint32_t *key = reinterpret_cast<uint32_t *>(ksm + (size_t)KP * 8);    // [C]
+    __shared__ uint32_t hist[256], wl[kSelThreads / 32], we[kSelThreads / 32];
+    __shared__ uint32_t s_prefix, s_kk;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const size_t e = blockIdx.x;
+    const float *Le = L + e * C;
+    for (int c = tid; c < C; c += kSelThreads) {
+        const float v = Le[c];
+        if (!isfinite(v)) atomicOr(err, kTopkBadLogit);
+        key[c] = desc_key(v);
     }
-    __syncthreads();
-    // bitonic sort, ascending keys
-    for (int size = 2; size <= CP; size <<= 1) {
+    for (int i = tid; i < KP; i += kSelThreads) sel[i] = ~0ull;
+    uint32_t prefix = 0u, mask = 0u, kk = (uint32_t)k;  // kk: rank sought among the prefix's keys
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        hist[tid] = 0u;
+        __syncthreads();
+        for (int c = tid; c < C; c += kSelThreads) {
+            const uint32_t kc = key[c];
+            if ((kc & mask) == prefix) atomicAdd(hist + ((kc >> shift) & 255u), 1u);
+        }
+        __syncthreads();
+        const uint32_t h = hist[tid];
+        uint32_t incl = h;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (lane == 31) wl[warp] = incl;
+        __syncthreads();
+        for (int w = 0; w < warp; ++w) incl += wl[w];
+        const uint32_t excl = incl - h;
+        if (excl < kk && kk <= incl) {
+            s_prefix = prefix | ((uint32_t)tid << shift);
+            s_kk = kk - excl;
+        }
+        __syncthreads();
+        prefix = s_prefix;
+        kk = s_kk;
+        mask |= 0xffu << shift;
+        __syncthreads();
+    }
+    // prefix = T; the k - kk keys below T all belong, then the first kk equal to T
+    const uint32_t T = prefix, nless = (uint32_t)k - kk;
+    uint32_t run_l = 0u, run_e = 0u;
+    const uint32_t lt = (1u << lane) - 1u;
+    for (int j0 = 0; j0 < C; j0 += kSelThreads) {
+        const int c = j0 + tid;
+        const uint32_t kc = c < C ? key[c] : 0xffffffffu;
+        const bool isl = c < C && kc < T, ise = c < C && kc == T;
+        const uint32_t bl = __ballot_sync(0xffffffffu, isl), be = __ballot_sync(0xffffffffu, ise);
+        if (lane == 0) {
+            wl[warp] = __popc(bl);
+            we[warp] = __popc(be);
+        }
+        __syncthreads();
+        uint32_t ol = run_l, oe = run_e, tl = 0u, te = 0u;
+        for (int w = 0; w < kSelThreads / 32; ++w) {
+            if (w < warp) {
+                ol += wl[w];
+                oe += we[w];
+            }
+            tl += wl[w];
+            te += we[w];
+        }
+        const unsigned long long k64 = ((unsigned long long)kc << 32) | (uint32_t)c;
+        if (isl) sel[ol + __popc(bl & lt)] = k64;
+        if (ise) {
+            const uint32_t r = oe + __popc(be & lt);
+            if (r < kk) sel[nless + r] = k64;
+        }
+        run_l += tl;
+        run_e += te;
+        __syncthreads();
+    }
+    // bitonic sort of the KP pairs, ascending keys (padding sorts last)
+    for (int size = 2; size <= KP; size <<= 1) {
         for (int stride = size >> 1; stride > 0; stride >>= 1) {
-            for (int i = threadIdx.x; i < CP / 2; i += kTrainThreads) {
+            for (int i = tid; i < KP / 2; i += kSelThreads) {
                 const int lo = 2 * i - (i & (stride - 1));  // pair (lo, lo + stride)
                 const int hi = lo + stride;
                 const bool up = (lo & size) == 0;
-                const unsigned long long a = keys[lo], b = keys[hi];
+                const unsigned long long a = sel[lo], b = sel[hi];
                 if ((a > b) == up) {
-                    keys[lo] = b;
-                    keys[hi] = a;
+                    sel[lo] = b;
+                    sel[hi] = a;
                 }
             }
             __syncthreads();
         }
     }
-    for (int i = threadIdx.x; i < k; i += kTrainThreads) {
-        const uint32_t c = (uint32_t)(keys[i] & 0xffffffffu);
-        idx_out[(size_t)e * k + i] = (int32_t)c;
-        lg_out[(size_t)e * k + i] = Le[c];
+    for (int i = tid; i < k; i += kSelThreads) {
+        const uint32_t c = (uint32_t)(sel[i] & 0xffffffffu);
+        idx_out[e * k + i] = (int32_t)c;
+        lg_out[e * k + i] = Le[c];
     }
 }
 
@@ -208,11 +279,13 @@ __global__ void __launch_bounds__(kTrainThreads) cov_grad_kernel(const float *__
 
 }  // namespace
 
-int topk_padded(int C) {
-    int cp = 1;
-    while (cp < C) cp <<= 1;
-    return cp;
+static int pow2_at_least(int v) {
+    int p = 1;
+    while (p < v) p <<= 1;
+    return p;
 }
+
+size_t topk_smem_bytes(int C, int k) { return (size_t)pow2_at_least(k) * 8 + (size_t)C * 4; }
 
 // Workspace of the support-maintenance calls: the error word, the row
 // statistics, u in double and g.
@@ -224,12 +297,13 @@ size_t train_ws_bytes(int R, int C) {
 
 cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float *lg,
                         uint32_t *err, cudaStream_t s) {
-    const int CP = topk_padded(C);
-    const size_t smem = (size_t)CP * 8;
-    cudaError_t e = cudaFuncSetAttribute(topk_rows_kernel,
+    if (R == 0) return cudaSuccess;
+    const int KP = pow2_at_least(k);
+    const size_t smem = topk_smem_bytes(C, k);
+    cudaError_t e = cudaFuncSetAttribute(topk_select_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    topk_rows_kernel<<<R, kTrainThreads, smem, s>>>(L, C, CP, k, idx, lg, err);
+    topk_select_kernel<<<(unsigned)R, kSelThreads, smem, s>>>(L, C, k, KP, idx, lg, err);
     return cudaGetLastError();
 }
 
