@@ -271,7 +271,8 @@ moce_status_t moce_mix(const void *x, int N, int H, int W, int C_in, int C_out, 
  *   V       device fp32 [C_in][d] (row c = channel embedding v_c)
  *   Q       device fp32 [C_out][d] (row e = expert embedding q_e)
  * (2 C_in d + d + C_out d router parameters, as the paper counts them.)
- * C_in <= 16384 (TopK sorts a row in shared memory), 1 <= d <= 4096.
+ * 4 C_in + 8 k' <= 227 KB, k' = k rounded up to a power of two (TopK keeps a
+ * row in shared memory: about 57,000 channels), 1 <= d <= 4096.
  * Non-finite logits give unspecified (but in-range) supports.
  *
  * moce_dynamic_workspace_bytes: device workspace of the dynamic calls
@@ -368,8 +369,10 @@ size_t moce_train_workspace_bytes(int C_in, int C_out);
  *   packed_idx    device int32 [C_out][k] out: the selected channels
  *   packed_logits device fp32 [C_out][k] out: their logits
  * SYNCHRONOUS (it validates): a non-finite logit returns
- * MOCE_ERR_BAD_SUPPORT (outputs then unspecified). C_in up to 16384
- * (MOCE_ERR_UNSUPPORTED beyond: one CTA sorts a row in shared memory).
+ * MOCE_ERR_BAD_SUPPORT (outputs then unspecified). Needs 4 C_in + 8 k' <=
+ * 227 KB, k' = k rounded up to a power of two (MOCE_ERR_UNSUPPORTED beyond:
+ * one CTA keeps a row's order keys in shared memory, selects the k-th by
+ * radix passes and sorts the k selected).
  */
 moce_status_t moce_topk_supports(const float *logits, int C_in, int C_out, int k,
                                  int32_t *packed_idx, float *packed_logits, void *ws,

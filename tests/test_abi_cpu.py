@@ -170,7 +170,7 @@ def test_dynamic_rejects_bad_arguments_on_host(lib):
     wb.argtypes, wb.restype = [I] * 7, S
     assert wb(2, 4, 4, 64, 8, 4, 16) > 0
     assert wb(2, 4, 4, 64, 8, 4, 0) == 0          # d < 1
-    assert wb(2, 4, 4, 20000, 8, 4, 16) == 0      # C_in beyond the shared-memory TopK
+    assert wb(2, 4, 4, 60000, 8, 4, 16) == 0      # C_in beyond the shared-memory TopK
     # the routing buffers do not depend on H, W: a larger H W only adds the forward part
     assert wb(2, 64, 64, 64, 8, 4, 16) > wb(2, 4, 4, 64, 8, 4, 16)
     f = lib.moce_forward_dynamic
@@ -192,7 +192,7 @@ def test_dynamic_rejects_bad_arguments_on_host(lib):
     assert call(ws=None) == 1
     assert call(wsb=64) == 1
     assert call(ws=ctypes.c_void_p(0x1080)) == 1     # not 256-byte aligned
-    assert call(C=20000, k=4) == 3                    # valid, TopK row does not fit
+    assert call(C=60000, k=4) == 3                    # valid, TopK row does not fit
     assert call(N=0) == 0
     m = lib.moce_mix
     m.argtypes = [P, I, I, I, I, I, I, I, I, P, P, P, I, P, P, P, S, P]
