@@ -51,6 +51,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="examples per layer instead of the workload's N (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto",
                     help="kernel path of the forward (auto, stream, steps)")
@@ -806,6 +808,8 @@ def main():
     args = parse_args()
     from paper_2608_23794_gb300 import synth
     cfg = synth.CONFIGS[args.workload]
+    if args.batch is not None:
+        cfg = cfg.replace(N=args.batch)
     if args.op == "train":
         run_train(args, cfg)
         return
