@@ -1,13 +1,14 @@
 // Support maintenance on the full routing matrix L [R][C] (training side):
 //
-//   topk_select_kernel    Eq. (support), Sec. 3.2: S_e = TopK(L_e, k), written in
-//                         deployment order (descending logit, equal logits by
+//   topk_warp_kernel,     Eq. (support), Sec. 3.2: S_e = TopK(L_e, k), written in
+//   topk_cta_kernel       deployment order (descending logit, equal logits by
 //                         ascending channel; -0.0 equals +0.0), so the result
-//                         is already packed. One CTA per row: a radix select of
-//                         the k-th order key (the key's high word orders the
-//                         logit), an ordered compaction of the k selected
-//                         (key, channel) pairs, then a bitonic sort of only
-//                         those, as 64-bit keys whose low word is the channel.
+//                         is already packed. One warp (many rows, small k) or
+//                         one CTA (few rows or large k) per row: a radix select
+//                         of the k-th order key, an ordered compaction of the
+//                         k selected (key, channel) pairs, then a bitonic sort
+//                         of only those, as 64-bit keys whose low word is the
+//                         channel.
 //   coverage kernels      Sec. 3.4: p_{e,c} = softmax(L_e)_c over all C channels,
 //                         u_c = (1/R) sum_e p_{e,c}, ubar = (1/C) sum_c u_c,
 //                         L_cov = sum_c (u_c - ubar)^2 / (ubar^2 + eps), and
@@ -70,6 +71,123 @@ __device__ double block_sum_d(double v, double *red) {
     return s;
 }
 
+// Shared memory of one warp's row: the KP selected pairs, 256 histogram bins
+// and the row's C order keys.
+__host__ __device__ inline size_t topk_warp_smem(int C, int k) {
+    int kp = 1;
+    while (kp < k) kp <<= 1;
+    return align_up((size_t)kp * 8 + 256 * 4 + (size_t)C * 4, 16);
+}
+
+// One row per warp (W warps per CTA, no block barriers): the row's C order
+// keys in the warp's shared memory; four 8-bit radix passes (a histogram of
+// 256 bins, a warp scan) find T, the k-th smallest key, and how many of the
+// keys equal to T are taken (the lowest channels first, as the tie rule
+// orders them); an ordered compaction by ballots (channel order) collects the
+// k selected (key, channel) pairs; a bitonic sort of those KP = k rounded up
+// to a power of two pairs gives deployment order.
+__global__ void __launch_bounds__(256) topk_warp_kernel(const float *__restrict__ L, int R,
+                                                          int C, int k, int KP,
+                                                          int32_t *__restrict__ idx_out,
+                                                          float *__restrict__ lg_out,
+                                                          uint32_t *err) {
+    extern __shared__ __align__(8) unsigned char ksm[];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const size_t per_warp = topk_warp_smem(C, k);
+    unsigned char *base = ksm + (size_t)w * per_warp;
+    unsigned long long *sel = reinterpret_cast<unsigned long long *>(base);   // [KP]
+    uint32_t *hist = reinterpret_cast<uint32_t *>(base + (size_t)KP * 8);    // [256]
+    uint32_t *key = hist + 256;                                               // [C]
+    const size_t e = (size_t)blockIdx.x * (blockDim.x >> 5) + w;
+    if (e >= (size_t)R) return;
+    const float *Le = L + e * C;
+    for (int c = lane; c < C; c += 32) {
+        const float v = Le[c];
+        if (!isfinite(v)) atomicOr(err, kTopkBadLogit);
+        key[c] = desc_key(v);
+    }
+    for (int i = lane; i < KP; i += 32) sel[i] = ~0ull;
+    uint32_t prefix = 0u, mask = 0u, kk = (uint32_t)k;  // kk: rank sought among the prefix's keys
+    for (int shift = 24; shift >= 0; shift -= 8) {
+#pragma unroll
+        for (int b = 0; b < 8; ++b) hist[lane * 8 + b] = 0u;
+        __syncwarp();
+        for (int c = lane; c < C; c += 32) {
+            const uint32_t kc = key[c];
+            if ((kc & mask) == prefix) atomicAdd(hist + ((kc >> shift) & 255u), 1u);
+        }
+        __syncwarp();
+        uint32_t hb[8], own = 0u;
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            hb[b] = hist[lane * 8 + b];
+            own += hb[b];
+        }
+        uint32_t incl = own;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        uint32_t run = incl - own, found = 0u, fb = 0u, fk = 0u;
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            if (!found && run < kk && kk <= run + hb[b]) {
+                found = 1u;
+                fb = (uint32_t)(lane * 8 + b);
+                fk = kk - run;
+            }
+            run += hb[b];
+        }
+        const int src = __ffs(__ballot_sync(0xffffffffu, found != 0u)) - 1;
+        fb = __shfl_sync(0xffffffffu, fb, src);
+        fk = __shfl_sync(0xffffffffu, fk, src);
+        prefix |= fb << shift;
+        kk = fk;
+        mask |= 0xffu << shift;
+        __syncwarp();
+    }
+    // prefix = T; the k - kk keys below T all belong, then the first kk equal to T
+    const uint32_t T = prefix, nless = (uint32_t)k - kk, lt = (1u << lane) - 1u;
+    uint32_t run_l = 0u, run_e = 0u;
+    for (int j0 = 0; j0 < C; j0 += 32) {
+        const int c = j0 + lane;
+        const uint32_t kc = c < C ? key[c] : 0xffffffffu;
+        const bool isl = c < C && kc < T, ise = c < C && kc == T;
+        const uint32_t bl = __ballot_sync(0xffffffffu, isl), be = __ballot_sync(0xffffffffu, ise);
+        const unsigned long long k64 = ((unsigned long long)kc << 32) | (uint32_t)c;
+        if (isl) sel[run_l + __popc(bl & lt)] = k64;
+        if (ise) {
+            const uint32_t r = run_e + __popc(be & lt);
+            if (r < kk) sel[nless + r] = k64;
+        }
+        run_l += __popc(bl);
+        run_e += __popc(be);
+    }
+    __syncwarp();
+    // bitonic sort of the KP pairs, ascending keys (padding sorts last)
+    for (int size = 2; size <= KP; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = lane; i < KP / 2; i += 32) {
+                const int lo = 2 * i - (i & (stride - 1));  // pair (lo, lo + stride)
+                const int hi = lo + stride;
+                const bool up = (lo & size) == 0;
+                const unsigned long long a = sel[lo], b = sel[hi];
+                if ((a > b) == up) {
+                    sel[lo] = b;
+                    sel[hi] = a;
+                }
+            }
+            __syncwarp();
+        }
+    }
+    for (int i = lane; i < k; i += 32) {
+        const uint32_t c = (uint32_t)(sel[i] & 0xffffffffu);
+        idx_out[e * k + i] = (int32_t)c;
+        lg_out[e * k + i] = Le[c];
+    }
+}
+
 // One row per CTA (256 threads): the row's C order keys in shared memory;
 // four 8-bit radix passes find T, the k-th smallest key, and how many of the
 // keys equal to T are taken (the lowest channels first, as the tie rule
@@ -77,7 +195,7 @@ __device__ double block_sum_d(double v, double *red) {
 // the k selected (key, channel) pairs; a bitonic sort of those KP = k rounded
 // up to a power of two pairs gives deployment order.
 constexpr int kSelThreads = 256;
-__global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float *__restrict__ L,
+__global__ void __launch_bounds__(kSelThreads) topk_cta_kernel(const float *__restrict__ L,
                                                                    int C, int k, int KP,
                                                                    int32_t *__restrict__ idx_out,
                                                                    float *__restrict__ lg_out,
@@ -285,7 +403,7 @@ static int pow2_at_least(int v) {
     return p;
 }
 
-size_t topk_smem_bytes(int C, int k) { return (size_t)pow2_at_least(k) * 8 + (size_t)C * 4; }
+size_t topk_smem_bytes(int C, int k) { return topk_warp_smem(C, k); }  // >= the CTA kernel's
 
 // Workspace of the support-maintenance calls: the error word, the row
 // statistics, u in double and g.
@@ -295,15 +413,31 @@ size_t train_ws_bytes(int R, int C) {
            align_up((size_t)C * 4, 256);
 }
 
+// Many rows with a small k (the per-example rows of the input-conditioned
+// variant) go one per warp; few rows or a large k one per CTA (more threads
+// per row for the sort, and every SM busy).
 cudaError_t launch_topk(const float *L, int R, int C, int k, int32_t *idx, float *lg,
                         uint32_t *err, cudaStream_t s) {
     if (R == 0) return cudaSuccess;
     const int KP = pow2_at_least(k);
-    const size_t smem = topk_smem_bytes(C, k);
-    cudaError_t e = cudaFuncSetAttribute(topk_select_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e;
+    if (KP <= 128 && R >= 8192) {
+        const size_t pw = topk_warp_smem(C, k);
+        int W = (int)((200 * 1024) / pw);  // rows (warps) per CTA
+        W = W < 1 ? 1 : (W > 8 ? 8 : W);
+        const size_t smem = pw * (size_t)W;
+        e = cudaFuncSetAttribute(topk_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+        if (e != cudaSuccess) return e;
+        topk_warp_kernel<<<(unsigned)((R + W - 1) / W), 32 * W, smem, s>>>(L, R, C, k, KP, idx, lg,
+                                                                           err);
+        return cudaGetLastError();
+    }
+    const size_t smem = (size_t)KP * 8 + (size_t)C * 4;
+    e = cudaFuncSetAttribute(topk_cta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
     if (e != cudaSuccess) return e;
-    topk_select_kernel<<<(unsigned)R, kSelThreads, smem, s>>>(L, C, k, KP, idx, lg, err);
+    topk_cta_kernel<<<(unsigned)R, kSelThreads, smem, s>>>(L, C, k, KP, idx, lg, err);
     return cudaGetLastError();
 }
 

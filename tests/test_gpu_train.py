@@ -47,6 +47,18 @@ def test_topk_bit_exact(moce, C, R, k, ties):
     assert np.array_equal(lg.cpu().numpy().view(np.uint32), rlg.view(np.uint32))
 
 
+@pytest.mark.parametrize("C,k", [(300, 20), (2048, 128), (96, 96), (33, 1)])
+@pytest.mark.parametrize("ties", [False, True])
+def test_topk_many_rows_bit_exact(moce, C, k, ties):
+    """9000 rows: the per-example row counts of the input-conditioned variant (one warp per
+    row for k <= 128) against the oracle."""
+    L = _logits(C, 9000, seed=C + k + 1, ties=ties)
+    idx, lg = moce.moce_topk_supports(torch.from_numpy(L).cuda(), k)
+    ridx, rlg = oracle.topk(L, k)
+    assert np.array_equal(idx.cpu().numpy(), ridx)
+    assert np.array_equal(lg.cpu().numpy().view(np.uint32), rlg.view(np.uint32))
+
+
 def test_topk_output_is_already_packed(moce):
     C, R, k = 256, 64, 16
     L = _logits(C, R, seed=3, ties=True)
