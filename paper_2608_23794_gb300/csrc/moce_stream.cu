@@ -76,6 +76,9 @@
 #ifndef MOCE_STREAM_PF
 #define MOCE_STREAM_PF 1
 #endif
+#ifndef MOCE_STREAM_GATES
+#define MOCE_STREAM_GATES 4
+#endif
 
 namespace moce {
 namespace {
@@ -1028,7 +1031,7 @@ constexpr int kLead = MOCE_STREAM_LEAD;
 // Items the pool producer prefetches into L2 ahead of its loads.
 constexpr int kPrefetch = MOCE_STREAM_PF;
 // SMs that run gates only.
-constexpr int kGateCtas = 4;
+constexpr int kGateCtas = MOCE_STREAM_GATES;
 
 bool plan_stream(int N, int HW, int C, int R, int k, int sms, StreamPlan *out) {
     if (C < 64 || C > 256 || C % 64 != 0 || R < 1 || R > kRMax || k < 1 || k > kKMax) return false;
