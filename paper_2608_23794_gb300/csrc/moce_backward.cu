@@ -281,23 +281,44 @@ __global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
     }
 }
 
+// Byte offset of the staged tables in a dx tile's shared memory (after the
+// R + 1 dy rows), and whether an example's tables (J weights, J row offsets,
+// C + 1 row pointers) are staged.
+__host__ __device__ inline size_t dx_tab_off(int R, int TP) {
+    return align_up((size_t)(R + 1) * TP * 2, 16);
+}
+inline size_t dx_tab_bytes(int J, int C) { return (size_t)J * 8 + (size_t)(C + 1) * 4; }
+constexpr size_t kDxTabMax = 96 * 1024;
+
 // dx of one tile, NHWC bf16 dy: lane = (channel c, chunk q of 8 positions);
 // the entries of c in increasing order (doff[m]: the entry's swizzled dy row
 // offset; am[n][m]: its weight a), then the residual expert and dz / HW.
 template <int TP>
 __global__ void __launch_bounds__(256) bwd_dx_nhwc_kernel(
     const uint16_t *__restrict__ dyT, int HW, int HWp, int C, int R, int J, int tiles,
-    const float *__restrict__ am, const int32_t *__restrict__ ptr, const int32_t *__restrict__ doff,
-    const uint8_t *__restrict__ inU, float inv_nU, const float *__restrict__ dz,
-    float *__restrict__ dx) {
+    const float *am, const int32_t *ptr, const int32_t *doff, const uint8_t *__restrict__ inU,
+    float inv_nU, const float *__restrict__ dz, float *__restrict__ dx, int tab) {
     constexpr int CPR = TP / 8;
     extern __shared__ __align__(16) unsigned char fsm[];
     unsigned char *ds = fsm;  // [R + 1][TP] bf16
     const int n = blockIdx.x / tiles, t = blockIdx.x - n * tiles;
     const int p0 = t * TP, np = min(TP, HW - p0);
     stage_dyT_rows<TP>(dyT + (size_t)n * (R + 1) * HWp + p0, HWp, R + 1, ds);
-    __syncthreads();
     const float *an = am + (size_t)n * J;
+    if (tab) {  // the example's tables fit: entry weights, row offsets and row pointers staged
+        float *tw = reinterpret_cast<float *>(fsm + dx_tab_off(R, TP));
+        int32_t *to = reinterpret_cast<int32_t *>(tw + J);
+        int32_t *tp = to + J;
+        for (int m = threadIdx.x; m < J; m += 256) {
+            tw[m] = __ldg(an + m);
+            to[m] = __ldg(doff + m);
+        }
+        for (int c = threadIdx.x; c <= C; c += 256) tp[c] = __ldg(ptr + c);
+        an = tw;
+        doff = to;
+        ptr = tp;
+    }
+    __syncthreads();
     const float inv_HW = 1.f / (float)HW;
     float *dxn = dx + ((size_t)n * HW + p0) * C;
     const uint32_t roff = (uint32_t)R * TP * 2 + ((uint32_t)swz_d(R, CPR) << 4);
@@ -308,23 +329,22 @@ __global__ void __launch_bounds__(256) bwd_dx_nhwc_kernel(
         const float base = dz[(size_t)n * C + c] * inv_HW;
 #pragma unroll
         for (int r = 0; r < 8; ++r) acc[r] = base;
-        const int m1 = __ldg(ptr + c + 1);
-        int m = __ldg(ptr + c);
+        const int m1 = ptr[c + 1];
+        int m = ptr[c];
         for (; m + 4 <= m1; m += 4) {  // four entries' loads in flight
             uint32_t of[4];
             float ww[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                of[u] = (uint32_t)__ldg(doff + m + u);
-                ww[u] = __ldg(an + m + u);
+                of[u] = (uint32_t)doff[m + u];
+                ww[u] = an[m + u];
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u)
                 fma8(acc, ww[u], *reinterpret_cast<const uint4 *>(ds + (of[u] ^ qx)));
         }
         for (; m < m1; ++m)
-            fma8(acc, __ldg(an + m),
-                 *reinterpret_cast<const uint4 *>(ds + ((uint32_t)__ldg(doff + m) ^ qx)));
+            fma8(acc, an[m], *reinterpret_cast<const uint4 *>(ds + ((uint32_t)doff[m] ^ qx)));
         if (inU[c]) fma8(acc, inv_nU, *reinterpret_cast<const uint4 *>(ds + (roff ^ qx)));
 #pragma unroll
         for (int r = 0; r < 8; ++r)
@@ -956,7 +976,10 @@ cudaError_t launch_backward(const void *x, const void *dy, int N, int HW, int C,
     bwd_dz_kernel<<<(unsigned)(((size_t)N * C + 255) / 256), 256, 0, s>>>(
         F(B.du), N, C, J, I(B.ptr), I(B.ent), F(B.dz));
     const float inv_nU = nU > 0 ? 1.f / (float)nU : 0.f;
-    const size_t smem_fx = (size_t)(R + 1) * kDxFastTile * 2;
+    const int tab = dx_tab_bytes(J, C) <= kDxTabMax &&
+                    dx_tab_off(R, kDxFastTile) + dx_tab_bytes(J, C) <= 227 * 1024 ? 1 : 0;
+    const size_t smem_fx =
+        tab ? dx_tab_off(R, kDxFastTile) + dx_tab_bytes(J, C) : (size_t)(R + 1) * kDxFastTile * 2;
     if (fast_dx) {
         bwd_gather_a_kernel<<<(unsigned)((rows * k + 255) / 256), 256, 0, s>>>(F(B.a), I(B.ent), N,
                                                                               J, F(B.am));
@@ -965,7 +988,8 @@ cudaError_t launch_backward(const void *x, const void *dy, int N, int HW, int C,
                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_fx);
         if (err != cudaSuccess) return err;
         bwd_dx_nhwc_kernel<kDxFastTile><<<(unsigned)((size_t)N * tiles_x), 256, smem_fx, s>>>(
-            dyT, HW, HWp, C, R, J, tiles_x, F(B.am), I(B.ptr), I(B.doff), inU, inv_nU, F(B.dz), dx);
+            dyT, HW, HWp, C, R, J, tiles_x, F(B.am), I(B.ptr), I(B.doff), inU, inv_nU, F(B.dz), dx,
+            tab);
         return cudaGetLastError();
     }
     const int tiles_x = (HW + TPX - 1) / TPX;
