@@ -154,22 +154,22 @@ __global__ void __launch_bounds__(256) bwd_dy_transpose_kernel(const uint16_t *_
 
 // Rows 0..E-1 of a TP-position tile from dyT (row stride HWp) into the
 // swizzled channel-major layout: 16-byte copies, four in flight per thread.
-template <int TP>
+template <int TP, int NT = 256>
 __device__ __forceinline__ void stage_dyT_rows(const uint16_t *__restrict__ src, int HWp, int E,
                                                unsigned char *ds) {
     constexpr int CPR = TP / 8;
     const int total = E * CPR;
-    for (int v0 = threadIdx.x; v0 < total; v0 += 4 * 256) {
+    for (int v0 = threadIdx.x; v0 < total; v0 += 4 * NT) {
         uint4 w[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const int v = v0 + u * 256, e = v / CPR, q = v % CPR;
+            const int v = v0 + u * NT, e = v / CPR, q = v % CPR;
             w[u] = v < total ? __ldg(reinterpret_cast<const uint4 *>(src + (size_t)e * HWp) + q)
                              : make_uint4(0u, 0u, 0u, 0u);
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const int v = v0 + u * 256, e = v / CPR, q = v % CPR;
+            const int v = v0 + u * NT, e = v / CPR, q = v % CPR;
             if (v < total)
                 *reinterpret_cast<uint4 *>(ds + (size_t)e * TP * 2 + ((q ^ swz_d(e, CPR)) << 4)) =
                     w[u];
@@ -189,12 +189,14 @@ __device__ __forceinline__ void stage_dyT_rows(const uint16_t *__restrict__ src,
 // lanes by a fixed shuffle tree. Channels come in decreasing entry count
 // (corder), so the lanes of a warp loop about equally long; which lane takes
 // a channel does not change its sums.
-template <int TP>
-__global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
+template <int TP, int NT>
+__global__ void __launch_bounds__(NT) bwd_da_nhwc_kernel(
     const uint16_t *__restrict__ x, const uint16_t *__restrict__ dyT, int HW, int HWp, int C,
     int R, int tiles, const int32_t *__restrict__ corder, const int32_t *__restrict__ ptr,
     const int2 *__restrict__ dtab, int J, float *__restrict__ part, float *__restrict__ psum) {
     constexpr int CPR = TP / 8;
+    // entries of a channel in flight per step: wide layers' channels have many
+    constexpr int kEU = TP == 64 ? 4 : 8;
     extern __shared__ __align__(16) unsigned char fsm[];
     unsigned char *xs = fsm;                       // [C][TP] bf16
     unsigned char *ds = fsm + (size_t)C * TP * 2;  // [R][TP] bf16
@@ -202,7 +204,7 @@ __global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
     const int p0 = t * TP, np = min(TP, HW - p0);
     const int C8 = C >> 3;
     const uint16_t *xn = x + ((size_t)n * HW + p0) * C;
-    for (int v = threadIdx.x; v < CPR * C8; v += 256) {
+    for (int v = threadIdx.x; v < CPR * C8; v += NT) {
         const int pg = v / C8, c8 = v - pg * C8;
         uint4 w[8];
 #pragma unroll
@@ -225,13 +227,13 @@ __global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
             *reinterpret_cast<uint4 *>(xs + (size_t)c * TP * 2 + ((pg ^ swz_x(c, CPR)) << 4)) = o;
         }
     }
-    stage_dyT_rows<TP>(dyT + (size_t)n * (R + 1) * HWp + p0, HWp, R, ds);
+    stage_dyT_rows<TP, NT>(dyT + (size_t)n * (R + 1) * HWp + p0, HWp, R, ds);
     __syncthreads();
     const int lane = threadIdx.x & 31, q = lane % CPR;
     constexpr int SPW = 32 / CPR;  // channels per warp step
     float *out = part + ((size_t)n * tiles + t) * (size_t)J;
     float *ps = psum + ((size_t)n * tiles + t) * C;
-    for (int sb = (threadIdx.x >> 5) * SPW; sb < C; sb += 8 * SPW) {
+    for (int sb = (threadIdx.x >> 5) * SPW; sb < C; sb += (NT / 32) * SPW) {
         const int sl = sb + lane / CPR;
         const bool valid = sl < C;
         const int c = valid ? __ldg(corder + sl) : 0;
@@ -249,14 +251,14 @@ __global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
         const int cnt = valid ? __ldg(ptr + c + 1) - m0 : 0;
         const int cmax = (int)__reduce_max_sync(0xffffffffu, (unsigned)cnt);
         const uint32_t qx = (uint32_t)q << 4;
-        for (int i = 0; i < cmax; i += 4) {
-            int2 tb[4];
-            float d[4];
+        for (int i = 0; i < cmax; i += kEU) {
+            int2 tb[kEU];
+            float d[kEU];
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+            for (int u = 0; u < kEU; ++u)
                 tb[u] = i + u < cnt ? __ldg(dtab + m0 + i + u) : make_int2(0, -1);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < kEU; ++u) {
                 const uint4 dv = *reinterpret_cast<const uint4 *>(ds + ((uint32_t)tb[u].x ^ qx));
                 float sm = bf16lo(dv.x) * xf[0];
                 sm = fmaf(bf16hi(dv.x), xf[1], sm);
@@ -271,10 +273,10 @@ __global__ void __launch_bounds__(256) bwd_da_nhwc_kernel(
 #pragma unroll
             for (int o = CPR / 2; o > 0; o >>= 1)
 #pragma unroll
-                for (int u = 0; u < 4; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
+                for (int u = 0; u < kEU; ++u) d[u] += __shfl_xor_sync(0xffffffffu, d[u], o);
             if (q == 0) {
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
+                for (int u = 0; u < kEU; ++u)
                     if (tb[u].y >= 0) out[tb[u].y] = d[u];
             }
         }
@@ -910,14 +912,15 @@ cudaError_t launch_backward(const void *x, const void *dy, int N, int HW, int C,
             cudaError_t e2 = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                   (int)smem);
             if (e2 != cudaSuccess) return e2;
-            kern<<<grid, 256, smem, s>>>((const uint16_t *)x, dyT, HW, HWp, C, R, tiles,
+            kern<<<grid, TPf == 64 ? 256 : 512, smem, s>>>((const uint16_t *)x, dyT, HW, HWp, C, R, tiles,
                                          I(B.corder), I(B.ptr),
                                          reinterpret_cast<const int2 *>(ws + B.dtab), J, F(B.part),
                                          F(B.psum));
             return cudaSuccess;
         };
-        err = TPf == 64 ? run(bwd_da_nhwc_kernel<64>)
-              : TPf == 32 ? run(bwd_da_nhwc_kernel<32>) : run(bwd_da_nhwc_kernel<16>);
+        // small tiles (wide layers) run one CTA per SM: 16 warps hide the table loads better
+        err = TPf == 64 ? run(bwd_da_nhwc_kernel<64, 256>)
+              : TPf == 32 ? run(bwd_da_nhwc_kernel<32, 512>) : run(bwd_da_nhwc_kernel<16, 512>);
         if (err != cudaSuccess) return err;
     } else {
         const size_t smem_da = (size_t)(C + R) * (B.TP + 1) * 4;
