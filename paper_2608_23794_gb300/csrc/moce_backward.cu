@@ -13,19 +13,28 @@
 //   dx_{p,c} = sum over (e, i) with S_e[i] = c of a_{e,i} dy_{p,e}
 //              + [c in U] dy_{p,R} / |U| + dz_c / HW
 // Kernels (every sum in a fixed order, so two calls give the same bits):
-//   bwd_da_kernel: per (example, tile of TP positions), x and dy staged as
-//     fp32 rows of TP (+1 padding) positions; thread per (e, i) pair -> the
-//     tile's partial da, thread per channel -> the tile's channel sums (the
-//     pool, fused, so x is read once); column sums over the tiles give da, z;
+//   the inverse support index first: a stable counting sort of the R k
+//     entries by channel (channel -> its (e, i) in increasing order), the
+//     channels in decreasing entry count, and per-entry tables (the entry's
+//     swizzled dy row offset in a tile, its index);
+//   dy transposed once to expert-major rows (bwd_dy_transpose_kernel);
+//   da and the pool, NHWC bf16 with C % 8 == 0 (bwd_da_nhwc_kernel): the x
+//     tile staged as swizzled channel-major bf16 rows by 16-byte loads and a
+//     register transpose; CPR lanes per channel hold the channel's positions
+//     in fp32 (their sum is the pool partial) and take the channel's entries
+//     one after another, each an 8-position dot product with the entry's dy
+//     row added over the lanes by a fixed shuffle tree; other layouts and
+//     dtypes: bwd_da_kernel (fp32 rows, a thread per (e, i) pair); column
+//     sums over the tiles give da and z;
 //   the gate: u gathered from z, hpre = W1 u + b1 and du = W1^T dh as tiled
 //     FP32 products over all N C_out rows; a warp per row between them for
 //     g, tau, the weights and the backward through the softmax, tau and the
 //     sigmoid;
 //   parameter gradients as fixed-order column sums over the rows (dW1 as a
 //     tiled product split over rows, then a column sum over the splits);
-//   the inverse support index (channel -> its (e, i) in increasing order),
-//     dz, then bwd_dx_kernel: per (example, tile), dy staged as fp32 rows,
-//     thread per channel accumulating its tile positions.
+//   dz from the inverse index; dx (bwd_dx_nhwc_kernel): lanes (channel, chunk
+//     of 8 positions) add the channel's entries from the staged dy rows, the
+//     residual row and dz / HW; other layouts and dtypes: bwd_dx_kernel.
 #include <math.h>
 
 #include "moce_internal.cuh"

@@ -3,7 +3,7 @@
 // inference: deterministic hard TopK, no noise). Per example n:
 //   h = ReLU(W_h z + b_h) in R^d                  router_hidden_kernel
 //   L_e(X)_c = L_{e,c} + sum_j q_{e,j} h_j v_{c,j}  dyn_logits_kernel
-//   S_e(X) = TopK(L_e(X), k), deployment order      topk_rows_kernel (moce_train.cu)
+//   S_e(X) = TopK(L_e(X), k), deployment order      launch_topk (moce_train.cu)
 //                                                   over the N C_out rows
 //   U(X) = channels no S_e(X) selects, ascending    dyn_resid_kernel
 // then the gate (Eq. (tau), reading z at S_e(X)) and the weights (Eq.
