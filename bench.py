@@ -479,30 +479,50 @@ def run_ours(args, cfg):
     dense_us = e0.elapsed_time(e1) * 1e3 / Kd
     dense_bytes = P * cfg.C_in * 2 + P * cfg.C_out * 2 + cfg.C_in * cfg.C_out * 2
 
-    # end to end through the public API: pinned host x -> device, forward, y -> pinned host
+    # end to end through the public API: pinned host x -> device, forward, y -> pinned host.
+    # Pipelined across steps: a copy stream brings step i + 1's x into the other device buffer
+    # while the compute stream runs step i's forward and reads its y back; every step's two
+    # copies are inside the timed region.
     x_host = bits.pin_memory()
-    y_host = torch.empty(ys[0].shape, dtype=torch.bfloat16).pin_memory()
-    x_dev, y_dev = xs[0], ys[0]
+    y_host = [torch.empty(ys[0].shape, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    x_dev, y_dev = [xs[0], xs[1 % n_rot]], [ys[0], ys[1 % n_rot]]
+    ws2 = [ws, moce.Workspace(cfg.N, cfg.H, cfg.W, cfg.C_in, cfg.C_out, cfg.k, device=dev)]
+    cs, ks = torch.cuda.Stream(device=dev), torch.cuda.current_stream()
+    ev_in = [torch.cuda.Event(), torch.cuda.Event()]
+    ev_done = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def e2e_run(K):
+        with torch.cuda.stream(cs):
+            cs.wait_stream(ks)
+            x_dev[0].copy_(x_host, non_blocking=True)
+            ev_in[0].record(cs)
+        for i in range(K):
+            b, nb = i & 1, (i & 1) ^ 1
+            if i + 1 < K:
+                with torch.cuda.stream(cs):
+                    if i >= 1:
+                        cs.wait_event(ev_done[nb])  # step i - 1 no longer reads x_dev[nb]
+                    x_dev[nb].copy_(x_host, non_blocking=True)
+                    ev_in[nb].record(cs)
+            ks.wait_event(ev_in[b])
+            moce.moce_forward(x_dev[b], "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max,
+                              ws=ws2[b], y=y_dev[b], path=args.path)
+            y_host[b].copy_(y_dev[b], non_blocking=True)
+            ev_done[b].record(ks)
+
     Ke = max(3, min(K, 200))
-    for _ in range(3):
-        x_dev.copy_(x_host, non_blocking=True)
-        moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
-                          y=y_dev, path=args.path)
-        y_host.copy_(y_dev, non_blocking=True)
+    e2e_run(3)
     torch.cuda.synchronize()
     e0.record()
-    for _ in range(Ke):
-        x_dev.copy_(x_host, non_blocking=True)
-        moce.moce_forward(x_dev, "nhwc", packed, W1, b1, w2, b2, cfg.tau_min, cfg.tau_max, ws=ws,
-                          y=y_dev, path=args.path)
-        y_host.copy_(y_dev, non_blocking=True)
+    e2e_run(Ke)
     e1.record()
     torch.cuda.synchronize()
     e2e_s = e0.elapsed_time(e1) * 1e-3 / Ke
     e2e_s = mdist.max_over_ranks(e2e_s, device=dev)
     e2e = {"value": mdist.job_throughput(nbytes, world, e2e_s) / 1e9, "unit": UNIT,
-           "h2d_bytes_per_step": x_bytes, "d2h_bytes_per_step": y_host.numel() * 2,
-           "us_per_layer": e2e_s * 1e6}
+           "h2d_bytes_per_step": x_bytes, "d2h_bytes_per_step": y_host[0].numel() * 2,
+           "us_per_layer": e2e_s * 1e6,
+           "note": "step i + 1's x copy overlaps step i's forward and y copy (two streams)"}
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
