@@ -153,3 +153,19 @@ def test_backward_dy_on_residual_only_reaches_unselected_channels():
     np.testing.assert_allclose(g.dx.cpu().numpy(), want, rtol=1e-6, atol=0)
     for f in ("dlogits", "dW1", "db1", "dw2", "db2"):
         assert float(getattr(g, f).abs().max()) == 0.0, f
+
+
+@pytest.mark.parametrize("cfg", [
+    LC("k_eq_c_empty_u", 2, 3, 5, 12, 4, 12, "f32", "nhwc", "relu", 12),     # |U| = 0
+    LC("one_expert", 3, 4, 4, 16, 1, 5, "f32", "nchw", "gelu", 16),          # R = 1
+    LC("one_channel_k1", 2, 3, 3, 1, 3, 1, "f32", "nhwc", "relu", 1),        # C = k = 1
+    LC("hw1_bf16", 5, 1, 1, 64, 7, 8, "bf16", "nhwc", "relu", 48),           # one position
+], ids=lambda c: c.name)
+def test_backward_degenerate_shapes(cfg):
+    g, ref, _ = _run(cfg, seed=7)
+    _close(g.dx.cpu().numpy(), ref["dx"], "dx")
+    _close(g.dlogits.cpu().numpy(), ref["dlogit"], "dlogits")
+    _close(g.dW1.cpu().numpy(), ref["dW1"], "dW1")
+    _close(g.db1.cpu().numpy(), ref["db1"], "db1")
+    _close(g.dw2.cpu().numpy(), ref["dw2"], "dw2")
+    _close(g.db2.cpu().numpy(), np.array([ref["db2"]]), "db2")

@@ -47,6 +47,11 @@ CASES = {
     "rn50_stage3_reduce": (CFG["rn50_stage3_reduce"].replace(N=2), 32),
     "vitb_ffn_exit_k32": (CFG["vitb_ffn_exit_k32"].replace(N=2), 32),
     "vitb_ffn_exit_k384": (CFG["vitb_ffn_exit_k384"].replace(N=1), 16),
+    # degenerate shapes: every channel selected (U(X) empty), a rank-1 router, a channel count
+    # that leaves a bitmap word partly unused, one example at one position
+    "k_eq_c": (LC("k_eq_c", 2, 3, 4, 24, 5, 24, "f32", "nhwc", "relu", 24), 4),
+    "d1_c70": (LC("d1_c70", 3, 5, 3, 70, 11, 6, "bf16", "nhwc", "gelu", 60), 1),
+    "n1_hw1": (LC("n1_hw1", 1, 1, 1, 40, 9, 3, "f32", "nchw", "relu", 30), 2),
 }
 
 
@@ -151,6 +156,7 @@ def _compare(cfg, d, seed=5):
 # fewest rows (of N C_out) whose set and order the bounds must decide, so that the exact
 # comparison is exercised (large k leaves many near-equal neighbours in a support)
 MIN_DECIDED = {"tiny_f32_nchw": 1.0, "ragged_bf16_nhwc": 1.0, "odd_f32_nhwc": 1.0,
+               "k_eq_c": 0.5, "d1_c70": 0.9, "n1_hw1": 1.0,
                "rn50_stage1_reduce": 0.8, "rn50_stage3_reduce": 0.1, "vitb_ffn_exit_k32": 0.05,
                "vitb_ffn_exit_k384": 0.0}
 
