@@ -244,7 +244,9 @@ moce_status_t moce_forward_noalloc(const void *x, int N, int H, int W, int C_in,
  *     resid_idx [C_in] with n_resid entries (as moce_forward);
  *   otherwise per-example supports, sup_idx [N][C_out][k], resid_idx
  *     [N][C_in] and n_resid_per_example [N] (device), as written by
- *     moce_dynamic_supports; n_resid is ignored.
+ *     moce_dynamic_supports; n_resid is ignored. A count outside [0, C_in]
+ *     is held to that range (the device cannot report it), so a row of
+ *     resid_idx is never read past its C_in entries.
  * ws: a forward workspace (moce_workspace_bytes). Asynchronous.
  */
 moce_status_t moce_mix(const void *x, int N, int H, int W, int C_in, int C_out, int k,
@@ -286,8 +288,9 @@ moce_status_t moce_mix(const void *x, int N, int H, int W, int C_in, int C_out, 
  * n_resid [N] (all device, int32 / fp32). Asynchronous.
  *
  * moce_forward_supports: the layer with given per-example supports (as
- * moce_dynamic_supports writes them): pool, gate and mix. ws: a forward
- * workspace (moce_workspace_bytes). Asynchronous.
+ * moce_dynamic_supports writes them): pool, gate and mix; n_resid counts
+ * are held to [0, C_in] as in moce_mix. ws: a forward workspace
+ * (moce_workspace_bytes). Asynchronous.
  *
  * moce_forward_dynamic: the whole variant: pool, router, TopK, U(X), gate and
  * mix. sup_idx, sup_logits, n_resid: optional device outputs (NULL: kept in

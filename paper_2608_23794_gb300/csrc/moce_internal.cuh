@@ -120,6 +120,12 @@ bool mix_geometry(int C, int R, int k, size_t smem_budget, MixGeom *g);
 struct PerExample {
     size_t sup_stride = 0, resid_stride = 0;
     const int32_t *nUa = nullptr;
+    // |U| of example n, held to [0, C]: a row of U has C entries, so a count
+    // outside that range (not one moce_dynamic_supports writes) reads no
+    // further than the row
+    __device__ __forceinline__ int count(int n, int nU, int C) const {
+        return nUa ? min(max(nUa[n], 0), C) : nU;
+    }
 };
 
 // ---------------------------------------------------------------- launchers (host)

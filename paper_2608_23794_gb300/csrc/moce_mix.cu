@@ -37,7 +37,7 @@ __global__ void __launch_bounds__(kThreads) mix_nchw_kernel(const T *__restrict_
     const int n = blockIdx.z;
     pidx += (size_t)n * pe.sup_stride;
     resid += (size_t)n * pe.resid_stride;
-    if (pe.nUa) nU = pe.nUa[n];
+    nU = pe.count(n, nU, C);
     const int e0 = blockIdx.y * EPB, e1 = min(R + 1, e0 + EPB);
     if (p >= HW) return;
     const T *xn = x + (size_t)n * C * HW + p;
@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(kThreads) mix_nhwc_generic_kernel(
             const float *ae = a + (n * R + e) * k;
             for (int i = 0; i < k; ++i) acc = fmaf(__ldg(ae + i), load_elem<T>(xp + __ldg(ie + i)), acc);
         } else {
-            const int nUn = pe.nUa ? pe.nUa[n] : nU;
+            const int nUn = pe.count((int)n, nU, C);
             const int32_t *rn = resid + n * pe.resid_stride;
             if (nUn > 0) {
                 for (int j = 0; j < nUn; ++j) acc += load_elem<T>(xp + __ldg(rn + j));
@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(kThreads) mix_nhwc_bf16_tiled_kernel(
     const int n = blockIdx.x / tiles, t = blockIdx.x - n * tiles;
     mix_nhwc_bf16_tile<GS>(msm, geom, x, HW, C, R, k, pidx + (size_t)n * pe.sup_stride,
                            a + (size_t)n * R * k, resid + (size_t)n * pe.resid_stride,
-                           pe.nUa ? pe.nUa[n] : nU, y, n, t);
+                           pe.count(n, nU, C), y, n, t);
 }
 
 template <int GS>

@@ -156,7 +156,7 @@ __global__ void __launch_bounds__(kWideThreads, 1) mix_wide_kernel(
     const float *an = a + (size_t)n * R * k;
     pidx += (size_t)n * pe.sup_stride;  // per-example supports (0: shared)
     resid += (size_t)n * pe.resid_stride;
-    if (pe.nUa) nU = pe.nUa[n];
+    nU = pe.count(n, nU, C);
     const int nch = (R + g.EB - 1) / g.EB;
     // table chunk j: the support indices, then the weights, of experts
     // j EB .. j EB + EB - 1 (each a contiguous run of rows in global memory)

@@ -241,3 +241,32 @@ def test_mix_entry_point_matches_the_step_path():
     y_mix = moce.moce_mix(dev["x"], cfg.layout, packed.packed_idx.view(cfg.C_out, cfg.k), a,
                           packed.resid_idx, packed.n_resid, ws)
     assert torch.equal(y_steps, y_mix)
+
+
+@pytest.mark.parametrize("dtype,layout,C", [("f32", "nchw", 40), ("f32", "nhwc", 40),
+                                            ("bf16", "nhwc", 72), ("bf16", "nhwc", 512)])
+def test_mix_holds_per_example_counts_to_the_row(dtype, layout, C):
+    """A per-example |U| above C_in mixes the whole row of C_in entries; one below 0 mixes none.
+
+    (Every mixing kernel: the NCHW one, the generic NHWC one, the tiled bf16 one and, from
+    512 channels, the wide one.)
+    """
+    from paper_2608_23794_gb300 import moce
+    N, H, W, R, k = 2, 5, 7, 9, 4
+    rng = np.random.default_rng(7)
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    shape = (N, C, H, W) if layout == "nchw" else (N, H, W, C)
+    x = torch.from_numpy(rng.standard_normal(shape).astype(np.float32)).to("cuda", tdt)
+    sidx = _cu(np.stack([rng.permutation(C)[: R * k].reshape(R, k) for _ in range(N)]), torch.int32)
+    a = _cu(rng.random((N, R, k)).astype(np.float32))
+    resid = _cu(np.stack([rng.permutation(C) for _ in range(N)]), torch.int32)
+    ws = moce.Workspace(N, H, W, C, R, k)
+    out = {}
+    for name, counts in (("held", [C + 50, -3]), ("in_range", [C, 0])):
+        out[name] = moce.moce_mix(x, layout, sidx, a, resid, _cu(np.array(counts), torch.int32), ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out["held"], out["in_range"])
+    yres = out["held"][..., R] if layout == "nhwc" else out["held"][:, R]
+    assert torch.count_nonzero(yres[1]) == 0
+    xm = x[0].float().mean(dim=-1 if layout == "nhwc" else 0)
+    assert torch.allclose(yres[0].float(), xm, atol=1e-2 if dtype == "bf16" else 1e-5)
