@@ -216,7 +216,8 @@ int moce_forward_path_launches(const void *x, int N, int H, int W, int C_in, int
     if (gate_smem_bytes(k) > 227 * 1024) return 0;
     switch (pick_path(x, N, H * W, C_in, C_out, k, dtype, layout, path)) {
         case MOCE_PATH_STREAM: return 1;
-        case MOCE_PATH_STEPS: return layout == MOCE_NHWC ? 4 : 3;  // [pool partials,] pool, gate, mix
+        case MOCE_PATH_STEPS:  // pool (one launch, or two with tile sums), gate, mix
+            return pool_launches(x, N, H * W, C_in, dtype, layout) + 2;
         default: return 0;
     }
 }

@@ -132,6 +132,16 @@ struct PerExample {
 cudaError_t launch_pack(int C, int R, int k, const int32_t *idx, const float *lg, int32_t *pidx,
                         float *plog, int32_t *resid, uint32_t *ws_words, cudaStream_t s);
 
+// Tiling of the NHWC pool (moce_pool.cu): vec channels per load, CB vectors
+// per CTA column block (chunks blocks), PT positions per span, spans spans per
+// example (1: z written directly; more: tile sums plus pool_finalize_kernel).
+struct PoolPlan {
+    int vec = 1, CB = 1, PT = 1, spans = 1;
+    unsigned chunks = 1;
+};
+PoolPlan pool_plan(const void *x, int N, int HW, int C, moce_dtype_t dt);
+// kernel launches of launch_pool for these arguments
+int pool_launches(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay);
 cudaError_t launch_pool(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay,
                         float *z, const WsLayout &L, unsigned char *ws, cudaStream_t s);
 

@@ -1,21 +1,56 @@
 // Global average pooling z = GAP(x) (Sec. 3.3), fp32 accumulation in a fixed
 // order so results are reproducible run to run.
 //
-// NHWC: pool_nhwc_partial_kernel reduces one tile of pool_px positions of one
-// example into per-channel partial sums (16-byte vector loads, one channel
-// vector per thread, several position rows per CTA reduced through shared
-// memory); pool_finalize_kernel adds the tile partials in tile order and
-// divides by H*W. NCHW: each channel plane is contiguous, one warp reduces a
-// plane with a fixed shuffle tree.
+// NHWC: pool_nhwc_kernel gives a CTA one example, one block of CB channel
+// vectors (16 bytes each: a warp reads 512 contiguous bytes of a position
+// row) and one span of positions; its rows = 256 / CB thread rows take every
+// rows-th position of the span, and the rows' sums are added in row order
+// through shared memory; a thread keeps kPoolU loads in flight. One span
+// per example (z written directly) when the (example, channel block) CTAs
+// fill half the GPU; otherwise enough spans to fill it, whose tile sums
+// pool_finalize_kernel adds in span order and divides by H*W. NCHW: each
+// channel plane is contiguous, one warp reduces a plane with a fixed shuffle
+// tree.
+#include <algorithm>
+
 #include "moce_internal.cuh"
 
 namespace moce {
 namespace {
 
+#ifndef MOCE_POOL_CTAS
+#define MOCE_POOL_CTAS (152 * 8)
+#endif
+#ifndef MOCE_POOL_HINT
+#define MOCE_POOL_HINT 1
+#endif
+constexpr long long kPoolCtas = MOCE_POOL_CTAS;  // one wave of 8 CTAs per SM
+
+#ifndef MOCE_POOL_UNROLL
+#define MOCE_POOL_UNROLL 8
+#endif
+constexpr int kPoolU = MOCE_POOL_UNROLL;  // loads in flight per thread
+
+// Vector loads of the NHWC pool: load() fetches one vector from a valid
+// address and zeroes it when ok is false (past the span: no branch, so a
+// thread's loads are all in flight), add() adds it to the channel sums.
 template <typename T, int VEC> struct VecLoad;
 template <> struct VecLoad<uint16_t, 8> {
-    static __device__ __forceinline__ void add(const uint16_t *p, float *acc) {
-        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(p));
+    using V = uint4;
+    static __device__ __forceinline__ V load(const uint16_t *p, bool ok) {
+        V v;
+#if MOCE_POOL_HINT
+        asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "l"(p));
+#else
+        v = __ldg(reinterpret_cast<const uint4 *>(p));
+#endif
+        const uint32_t m = ok ? 0xffffffffu : 0u;
+        v.x &= m; v.y &= m; v.z &= m; v.w &= m;
+        return v;
+    }
+    static __device__ __forceinline__ void add(const V &v, float *acc) {
         acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x);
         acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
         acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z);
@@ -23,63 +58,70 @@ template <> struct VecLoad<uint16_t, 8> {
     }
 };
 template <> struct VecLoad<float, 4> {
-    static __device__ __forceinline__ void add(const float *p, float *acc) {
+    using V = float4;
+    static __device__ __forceinline__ V load(const float *p, bool ok) {
         const float4 v = __ldg(reinterpret_cast<const float4 *>(p));
+        return ok ? v : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    static __device__ __forceinline__ void add(const V &v, float *acc) {
         acc[0] += v.x; acc[1] += v.y; acc[2] += v.z; acc[3] += v.w;
     }
 };
 template <typename T> struct VecLoad<T, 1> {
-    static __device__ __forceinline__ void add(const T *p, float *acc) { acc[0] += load_elem<T>(p); }
+    using V = float;
+    static __device__ __forceinline__ V load(const T *p, bool ok) {
+        const float v = load_elem<T>(p);
+        return ok ? v : 0.f;
+    }
+    static __device__ __forceinline__ void add(const V &v, float *acc) { acc[0] += v; }
 };
 
-// grid (pool_tiles, N); partial[(n*tiles + t)*C + c]
+// grid (chunks, spans, N). Thread (row, cvl): channel vector ch CB + cvl,
+// positions p0 + row, p0 + row + rows, ... of the span. One span: z[n][c]
+// = sum / HW; otherwise partial[(n spans + t) C + c] = the span's sum.
 template <typename T, int VEC>
-__global__ void __launch_bounds__(kThreads) pool_nhwc_partial_kernel(const T *__restrict__ x, int HW,
-                                                                     int C, int PP, int tiles,
-                                                                     float *__restrict__ partial) {
-    __shared__ float red[kThreads * VEC];
-    const int n = blockIdx.y, t = blockIdx.x;
-    const int p0 = t * PP, p1 = min(HW, p0 + PP);
-    const int V = C / VEC;
-    const int span = V < kThreads ? V : kThreads;
-    const int rows = kThreads / span;
-    const int row = threadIdx.x / span, cvl = threadIdx.x % span;
-    const T *xe = x + (size_t)n * HW * C;
-    float *out = partial + ((size_t)n * tiles + t) * C;
-    for (int cv0 = 0; cv0 < V; cv0 += span) {
-        const int cv = cv0 + cvl;
-        float acc[VEC];
+__global__ void __launch_bounds__(kThreads) pool_nhwc_kernel(const T *__restrict__ x, int HW, int C,
+                                                             int CB, int PT, int spans,
+                                                             float *__restrict__ partial,
+                                                             float *__restrict__ z) {
+    __shared__ float red[kThreads * VEC];  // [row][j][cvl]
+    const int ch = blockIdx.x, t = blockIdx.y, n = blockIdx.z;
+    const int V = C / VEC, rows = kThreads / CB;
+    const int row = threadIdx.x / CB, cvl = threadIdx.x - row * CB;
+    const int cv = ch * CB + cvl;
+    const int p0 = t * PT, p1 = min(HW, p0 + PT);
+    float acc[VEC];
 #pragma unroll
-        for (int j = 0; j < VEC; ++j) acc[j] = 0.f;
-        if (row < rows && cv < V) {
-            const T *col = xe + (size_t)cv * VEC;
-            int p = p0 + row;
-            for (; p + 3 * rows < p1; p += 4 * rows) {
-                VecLoad<T, VEC>::add(col + (size_t)p * C, acc);
-                VecLoad<T, VEC>::add(col + (size_t)(p + rows) * C, acc);
-                VecLoad<T, VEC>::add(col + (size_t)(p + 2 * rows) * C, acc);
-                VecLoad<T, VEC>::add(col + (size_t)(p + 3 * rows) * C, acc);
+    for (int j = 0; j < VEC; ++j) acc[j] = 0.f;
+    if (row < rows && cv < V) {
+        using L = VecLoad<T, VEC>;
+        const T *col = x + (size_t)n * HW * C + (size_t)cv * VEC;
+        // kPoolU loads in flight (the last batch predicated), added in
+        // position order
+        for (int p = p0 + row; p < p1; p += kPoolU * rows) {
+            typename L::V v[kPoolU];
+#pragma unroll
+            for (int u = 0; u < kPoolU; ++u) {
+                const int pu = p + u * rows;
+                v[u] = L::load(col + (size_t)(pu < p1 ? pu : p) * C, pu < p1);
             }
-            for (; p < p1; p += rows) VecLoad<T, VEC>::add(col + (size_t)p * C, acc);
+#pragma unroll
+            for (int u = 0; u < kPoolU; ++u) L::add(v[u], acc);
         }
-        if (rows == 1) {
-            if (cv < V) {
+    }
+    if (row < rows) {
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) out[(size_t)cv * VEC + j] = acc[j];
-            }
-        } else {
-            if (row < rows) {
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) red[(row * span + cvl) * VEC + j] = acc[j];
-            }
-            __syncthreads();
-            for (int q = threadIdx.x; q < span * VEC; q += kThreads) {
-                float s = 0.f;
-                for (int r = 0; r < rows; ++r) s += red[r * span * VEC + q];
-                out[(size_t)cv0 * VEC + q] = s;
-            }
-            __syncthreads();
-        }
+        for (int j = 0; j < VEC; ++j) red[(row * VEC + j) * CB + cvl] = acc[j];
+    }
+    __syncthreads();
+    for (int q = threadIdx.x; q < CB * VEC; q += kThreads) {
+        const int j = q / CB, v = ch * CB + (q - j * CB);
+        if (v >= V) continue;
+        float s = 0.f;
+        for (int r = 0; r < rows; ++r) s += red[r * VEC * CB + q];
+        const size_t c = (size_t)v * VEC + j;
+        if (spans == 1) z[(size_t)n * C + c] = s / (float)HW;
+        else partial[((size_t)n * spans + t) * C + c] = s;
     }
 }
 
@@ -112,9 +154,37 @@ __global__ void __launch_bounds__(kThreads) pool_nchw_kernel(const T *__restrict
 
 }  // namespace
 
+PoolPlan pool_plan(const void *x, int N, int HW, int C, moce_dtype_t dt) {
+    PoolPlan pp;
+    const bool aligned = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+    pp.vec = dt == MOCE_BF16 ? (aligned && C % 8 == 0 ? 8 : 1) : (aligned && C % 4 == 0 ? 4 : 1);
+    const int V = C / pp.vec;
+    pp.CB = V < 32 ? V : 32;
+    const int rows = kThreads / pp.CB;
+    pp.chunks = (unsigned)((V + pp.CB - 1) / pp.CB);
+    // spans per example: one (z written directly, no second launch) once the
+    // (example, channel block) CTAs alone reach half a wave; otherwise about
+    // kPoolCtas CTAs in all, at most one span per thread row of positions and
+    // no more than the workspace's tile partials (ws_layout's pool_tiles)
+    const long long base = (long long)N * pp.chunks;
+    const int px = pool_tile_px(C), tiles = (HW + px - 1) / px;
+    long long spans = 2 * base >= kPoolCtas ? 1 : (kPoolCtas + base - 1) / base;
+    spans = std::min<long long>(spans, std::min<long long>(tiles, (HW + rows - 1) / rows));
+    spans = std::max<long long>(1, std::min<long long>(spans, 65535));  // a grid dimension
+    pp.PT = (int)((HW + spans - 1) / spans);
+    pp.spans = (HW + pp.PT - 1) / pp.PT;
+    return pp;
+}
+
+int pool_launches(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay) {
+    if (N == 0 || HW <= 0) return 0;
+    if (lay == MOCE_NCHW) return 1;
+    return pool_plan(x, N, HW, C, dt).spans > 1 ? 2 : 1;
+}
+
 cudaError_t launch_pool(const void *x, int N, int HW, int C, moce_dtype_t dt, moce_layout_t lay,
                         float *z, const WsLayout &L, unsigned char *ws, cudaStream_t s) {
-    if (N == 0) return cudaSuccess;
+    if (N == 0 || HW <= 0) return cudaSuccess;
     if (lay == MOCE_NCHW) {
         const size_t planes = (size_t)N * C;
         const unsigned grid = (unsigned)((planes + 7) / 8);
@@ -125,26 +195,31 @@ cudaError_t launch_pool(const void *x, int N, int HW, int C, moce_dtype_t dt, mo
         return cudaGetLastError();
     }
     float *partial = reinterpret_cast<float *>(ws + L.partial);
-    const dim3 grid(L.pool_tiles, N);
-    const bool aligned = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+    const PoolPlan pp = pool_plan(x, N, HW, C, dt);
+    const int VEC = pp.vec, CB = pp.CB, PT = pp.PT, S = pp.spans;
+    const unsigned chunks = pp.chunks;
+    if (S > L.pool_tiles) return cudaErrorInvalidValue;  // the tile sums would not fit
+    const dim3 grid(chunks, (unsigned)S, (unsigned)N);
     if (dt == MOCE_BF16) {
-        if (aligned && C % 8 == 0)
-            pool_nhwc_partial_kernel<uint16_t, 8><<<grid, kThreads, 0, s>>>(
-                (const uint16_t *)x, HW, C, L.pool_px, L.pool_tiles, partial);
+        if (VEC == 8)
+            pool_nhwc_kernel<uint16_t, 8><<<grid, kThreads, 0, s>>>((const uint16_t *)x, HW, C, CB,
+                                                                    PT, S, partial, z);
         else
-            pool_nhwc_partial_kernel<uint16_t, 1><<<grid, kThreads, 0, s>>>(
-                (const uint16_t *)x, HW, C, L.pool_px, L.pool_tiles, partial);
+            pool_nhwc_kernel<uint16_t, 1><<<grid, kThreads, 0, s>>>((const uint16_t *)x, HW, C, CB,
+                                                                    PT, S, partial, z);
     } else {
-        if (aligned && C % 4 == 0)
-            pool_nhwc_partial_kernel<float, 4><<<grid, kThreads, 0, s>>>(
-                (const float *)x, HW, C, L.pool_px, L.pool_tiles, partial);
+        if (VEC == 4)
+            pool_nhwc_kernel<float, 4><<<grid, kThreads, 0, s>>>((const float *)x, HW, C, CB, PT, S,
+                                                                 partial, z);
         else
-            pool_nhwc_partial_kernel<float, 1><<<grid, kThreads, 0, s>>>(
-                (const float *)x, HW, C, L.pool_px, L.pool_tiles, partial);
+            pool_nhwc_kernel<float, 1><<<grid, kThreads, 0, s>>>((const float *)x, HW, C, CB, PT, S,
+                                                                 partial, z);
     }
-    const size_t nz = (size_t)N * C;
-    pool_finalize_kernel<<<(unsigned)((nz + kThreads - 1) / kThreads), kThreads, 0, s>>>(
-        partial, N, C, L.pool_tiles, HW, z);
+    if (S > 1) {
+        const size_t nz = (size_t)N * C;
+        pool_finalize_kernel<<<(unsigned)((nz + kThreads - 1) / kThreads), kThreads, 0, s>>>(
+            partial, N, C, S, HW, z);
+    }
     return cudaGetLastError();
 }
 

@@ -115,14 +115,19 @@ def test_forward_path_selection_on_host(lib):
     assert call(1, 6) == 3
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 6) == 0
     assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 6) is None
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 4   # pool partials, pool, gate, mix
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == 3   # pool (one span per example), gate, mix
     assert name(fake, 2, 8, 8, 64, 16, 4, 1, 0, 0) == b"pool+gate+mix"
-    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
+    assert n(fake, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 3
+    # two examples of 56 x 56 positions: the pool splits each into spans whose tile sums a
+    # second kernel adds
+    assert n(fake, 2, 56, 56, 256, 16, 4, 1, 0, 4) == 4
+    # 160 examples of 7 x 7 x 1024: enough CTAs with one span per example
+    assert n(fake, 160, 7, 7, 1024, 16, 4, 1, 0, 4) == 3
     # fp32 has no stream kernel either; the steps run any dtype, layout and alignment
     assert call(0, 6) == 3
     odd = ctypes.c_void_p(0x1002)
     assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 6) == 0
-    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 4
+    assert n(odd, 2, 8, 8, 64, 16, 4, 1, 0, 4) == 3
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 6) == 0
     assert n(fake, 2, 8, 8, 64, 16, 4, 1, 1, 0) == 3   # NCHW: pool, gate, mix
 

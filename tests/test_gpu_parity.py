@@ -128,6 +128,39 @@ def test_pool_and_gate(name):
     np.testing.assert_allclose(a.cpu().numpy(), aref, rtol=2e-5, atol=1e-7)
 
 
+POOL_SHAPES = {
+    # (N, H, W, C, dtype, element offset of x): the tilings of the NHWC pool
+    "many_spans_c256": (2, 56, 56, 256, "bf16", 0),
+    "spans_capped_c2048": (3, 7, 7, 2048, "bf16", 0),
+    "spans_c3072": (2, 14, 14, 3072, "bf16", 0),
+    "five_spans_c1024": (70, 14, 14, 1024, "bf16", 0),
+    "one_span_c1024": (160, 7, 7, 1024, "bf16", 0),
+    "narrow_block_f32": (3, 5, 7, 60, "f32", 0),
+    "narrow_block_bf16": (2, 9, 11, 72, "bf16", 0),
+    "scalar_ragged_block": (2, 6, 6, 70, "bf16", 0),
+    "unaligned_bf16": (2, 8, 8, 256, "bf16", 1),
+    "unaligned_f32": (2, 8, 8, 128, "f32", 1),
+    "one_position": (1, 1, 1, 8, "bf16", 0),
+}
+
+
+@pytest.mark.parametrize("name", list(POOL_SHAPES))
+def test_pool_tilings(name):
+    """z = GAP(x) against the oracle for one span and several per example, 16-byte and
+    scalar loads, channel blocks narrower than 32 vectors and a ragged last block."""
+    from paper_2608_23794_gb300 import moce
+    N, H, W, C, dt, off = POOL_SHAPES[name]
+    tdt = torch.bfloat16 if dt == "bf16" else torch.float32
+    rng = np.random.default_rng(17)
+    xf = rng.standard_normal((N, H, W, C)).astype(np.float32)
+    buf = torch.empty(N * H * W * C + off, dtype=tdt, device="cuda")
+    x = buf[off:].view(N, H, W, C)
+    x.copy_(torch.from_numpy(xf))
+    z = moce.moce_pool(x, "nhwc").cpu().numpy()
+    zref = oracle.pool(x.float().cpu().numpy(), "nhwc")
+    np.testing.assert_allclose(z, zref, rtol=1e-5, atol=1e-6)
+
+
 # ------------------------------------------------------------------ forward, element by element
 
 
