@@ -93,6 +93,32 @@ def fp32_fma_peak(sms: int, mhz: float) -> float:
     return FP32_LANES_PER_SM * sms * mhz * 1e6
 
 
+def sgemm_fma_rate(dev) -> float:
+    """FP32 multiply-adds per second of cuBLAS SGEMM (8192^3 at the "highest" float32 matmul
+    precision: no TF32), a measured check beside the derived FP32 peak."""
+    import torch
+    n = 8192
+    g = torch.Generator(device=dev).manual_seed(0)
+    a = torch.randn(n, n, device=dev, generator=g)
+    b = torch.randn(n, n, device=dev, generator=g)
+    c = torch.empty(n, n, device=dev)
+    prec = torch.get_float32_matmul_precision()
+    torch.set_float32_matmul_precision("highest")
+    try:
+        for _ in range(3):
+            torch.matmul(a, b, out=c)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(10):
+            torch.matmul(a, b, out=c)
+        e1.record()
+        torch.cuda.synchronize()
+    finally:
+        torch.set_float32_matmul_precision(prec)
+    return n ** 3 / (e0.elapsed_time(e1) * 1e-3 / 10)
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -462,6 +488,10 @@ def run_ours(args, cfg):
                                    f"{props.multi_processor_count} SMs x "
                                    f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
                     "kernel": kern_label, "algorithmic_macs_per_launch": macs}
+        sgemm = sgemm_fma_rate(dev)
+        roofline["sgemm_check"] = {"value": sgemm / 1e12, "unit": "T FMA/s",
+                                   "frac_of_derived_peak": sgemm / fma_peak,
+                                   "what": "cuBLAS SGEMM 8192^3, no TF32"}
     floors = {"hbm_us": hbm_floor * 1e6, "fp32_fma_us": fma_floor * 1e6,
               "binding": roofline["bound"], "measured_us": kern_s * 1e6,
               "frac_of_binding": max(hbm_floor, fma_floor) / kern_s}
