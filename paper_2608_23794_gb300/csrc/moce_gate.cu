@@ -6,9 +6,11 @@
 // gate_tiled_kernel (k a multiple of 16): the hidden layer of the gate of
 // every expert of one example is the product H = U W1^T (U [R][k]: row e =
 // z[n, S_e] in deployment order; W1 [k][k], shared by every expert), a dense
-// contraction. One CTA of 256 threads takes 64 experts: U^T [k][64] is
-// gathered into shared memory, W1^T streams through it in chunks of KC
-// inputs, and thread (te, th) accumulates experts 4 te .. 4 te + 3 times
+// contraction. One CTA of 256 threads takes 64 experts: z of the example is
+// staged once; then, in chunks of KC = 32 inputs, the chunk's support
+// indices, its rows of U^T [KC][64] (gathered from z) and of W1^T [KC][k]
+// pass through shared memory (about 42 KB at k = 128, so several CTAs share
+// an SM), and thread (te, th) accumulates experts 4 te .. 4 te + 3 times
 // hidden units TN th .. TN th + TN - 1 (TN = k / 16) in registers, over the
 // inputs in order (fma.rn.f32x2 on pairs of hidden units). Each expert's 16
 // partial sums w2 . ReLU(h + b1) are added by shuffles in a fixed order; then
@@ -32,19 +34,14 @@ __global__ void __launch_bounds__(kThreads) gate_kernel(
 constexpr int kTE = 64;        // experts per tiled-gate CTA
 constexpr int kUS = kTE + 4;   // padded row of U^T (float4-aligned, rows 4 banks apart)
 
-__host__ __device__ inline int tiled_kc(int k) {
-    int kc = 24576 / k;  // W1^T chunk of at most 96 KB
-    if (kc > k) kc = k;
-    return kc & ~3;
-}
-// Floats of the W1^T buffer, which first holds z of the example and the
-// CTA's block of support indices (C floats plus kTE rows of k + 1 indices).
-__host__ __device__ inline size_t tiled_wt(int k, int C) {
-    const size_t a = (size_t)tiled_kc(k) * k, b = (size_t)C + (size_t)kTE * (k + 1);
-    return a > b ? a : b;
-}
+constexpr int kKC = 32;        // inputs per chunk of the tiled gate
+
+// Floats of the tiled gate's shared memory: U^T and W1^T chunks, tau, the
+// chunk's index rows (KC + 1 apart: the gather reads them without bank
+// conflicts) and z of the example.
 __host__ __device__ inline size_t tiled_smem(int k, int C) {
-    return ((size_t)k * kUS + tiled_wt(k, C) + kTE) * sizeof(float);
+    return ((size_t)kKC * kUS + (size_t)kKC * k + kTE + (size_t)kTE * (kKC + 1) + (size_t)C) *
+           sizeof(float);
 }
 
 template <int TN>
@@ -57,35 +54,17 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
     pidx += (size_t)blockIdx.y * sup_stride;  // per-example supports (0: shared)
     plog += (size_t)blockIdx.y * sup_stride;
     extern __shared__ __align__(16) float tsm[];
-    const int KC = tiled_kc(k);
-    float *Ut = tsm;                      // [k][kUS]: Ut[i][el] = z[n, S_(e0 + el)][i]
-    float *Wt = Ut + (size_t)k * kUS;     // [KC][k]: Wt[i][j] = W1[j][i0 + i]
-    float *tau_s = Wt + tiled_wt(k, C);   // [kTE]
+    float *Ut = tsm;                                   // [KC][kUS]: Ut[i][el] = z[n, S_(e0+el)][i0+i]
+    float *Wt = Ut + (size_t)kKC * kUS;                // [KC][k]: Wt[i][j] = W1[j][i0 + i]
+    float *tau_s = Wt + (size_t)kKC * k;               // [kTE]
+    int32_t *is = reinterpret_cast<int32_t *>(tau_s + kTE);  // [kTE][KC + 1]
+    float *zs = reinterpret_cast<float *>(is + kTE * (kKC + 1));  // [C]
     const int n = blockIdx.y, e0 = blockIdx.x * kTE;
     const int tid = threadIdx.x, te = tid >> 4, th = tid & 15;
-    const float *zn = z + (size_t)n * C;
-
+    const int ne = min(kTE, R - e0);
     {
-        // stage z_n and the block's support indices (coalesced loads; index
-        // rows of k + 1 so that the gather below reads them without bank
-        // conflicts), then gather U^T with consecutive threads on consecutive
-        // experts (conflict-free stores)
-        float *zs = Wt;
-        int32_t *is = reinterpret_cast<int32_t *>(Wt + C);
-        const int ne = min(kTE, R - e0);
+        const float *zn = z + (size_t)n * C;
         for (int c = tid; c < C; c += 256) zs[c] = __ldcg(zn + c);
-        const int4 *src = reinterpret_cast<const int4 *>(pidx + (size_t)e0 * k);
-        for (int q = tid; q < ne * k / 4; q += 256) {
-            const int4 v = __ldg(src + q);
-            const int el = (4 * q) / k, i = 4 * q - el * k;
-            int32_t *d = is + (size_t)el * (k + 1) + i;
-            d[0] = v.x; d[1] = v.y; d[2] = v.z; d[3] = v.w;
-        }
-        __syncthreads();
-        for (int q = tid; q < kTE * k; q += 256) {
-            const int el = q & (kTE - 1), i = q / kTE;
-            Ut[i * kUS + el] = el < ne ? zs[is[el * (k + 1) + i]] : 0.f;
-        }
     }
     // thread th's hidden units, in pairs: pair p < 2 (TN / 4) is units
     // 64 (p / 2) + 4 th + 2 (p mod 2) + {0, 1}; a last pair (TN mod 4 = 2) is
@@ -100,9 +79,15 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
     for (int m = 0; m < 4; ++m)
 #pragma unroll
         for (int p = 0; p < NP; ++p) acc[m][p] = make_float2(0.f, 0.f);
-    for (int i0 = 0; i0 < k; i0 += KC) {
-        const int kc = min(KC, k - i0);
-        __syncthreads();  // U ready / the previous chunk consumed
+    for (int i0 = 0; i0 < k; i0 += kKC) {
+        const int kc = min(kKC, k - i0);
+        __syncthreads();  // z staged / the previous chunk consumed
+        // the chunk's support indices (consecutive threads on consecutive
+        // inputs of an expert: coalesced loads, conflict-free stores)
+        for (int q = tid; q < ne * kc; q += 256) {
+            const int el = q / kc, i = q - el * kc;
+            is[el * (kKC + 1) + i] = __ldg(pidx + (size_t)(e0 + el) * k + i0 + i);
+        }
         // Wt[i][j] = W1[j][i0 + i]: a thread reads 4 inputs of one hidden unit
 #pragma unroll 4
         for (int q = tid; q < k * (kc >> 2); q += 256) {
@@ -114,9 +99,16 @@ __global__ void __launch_bounds__(256) gate_tiled_kernel(
             Wt[(4 * i4 + 3) * k + j] = w.w;
         }
         __syncthreads();
+        // U^T rows of the chunk, consecutive threads on consecutive experts
+        // (conflict-free stores); experts past R read as zero
+        for (int q = tid; q < kTE * kc; q += 256) {
+            const int el = q & (kTE - 1), i = q / kTE;
+            Ut[i * kUS + el] = el < ne ? zs[is[el * (kKC + 1) + i]] : 0.f;
+        }
+        __syncthreads();
 #pragma unroll 2
         for (int i = 0; i < kc; ++i) {
-            const float4 u = *reinterpret_cast<const float4 *>(Ut + (size_t)(i0 + i) * kUS + 4 * te);
+            const float4 u = *reinterpret_cast<const float4 *>(Ut + (size_t)i * kUS + 4 * te);
             const float *wr = Wt + (size_t)i * k;
             float2 w[NP];
 #pragma unroll
