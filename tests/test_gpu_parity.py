@@ -128,6 +128,35 @@ def test_pool_and_gate(name):
     np.testing.assert_allclose(a.cpu().numpy(), aref, rtol=2e-5, atol=1e-7)
 
 
+GATE_BLOCKS = {
+    # C_out not a multiple of the tiled gate's 64-expert block, k on its tiled path, C_in ragged
+    "r70_k32": synth.LayerConfig("r70_k32", 3, 2, 2, 200, 70, 32, "bf16", "nhwc", "relu", 180),
+    "r5_k64": synth.LayerConfig("r5_k64", 2, 2, 2, 300, 5, 64, "bf16", "nhwc", "gelu", 256),
+    "r130_k128": synth.LayerConfig("r130_k128", 2, 2, 2, 256, 130, 128, "bf16", "nhwc", "relu", 224),
+    "r100_k384": synth.LayerConfig("r100_k384", 1, 1, 1, 512, 100, 384, "bf16", "nhwc", "gelu", 448),
+}
+
+
+@pytest.mark.parametrize("name", list(GATE_BLOCKS))
+def test_tiled_gate_partial_expert_blocks(name):
+    """tau and the weights against the oracle when the last block of 64 experts is partial."""
+    from paper_2608_23794_gb300 import moce
+    cfg = GATE_BLOCKS[name]
+    lay = synth.make_layer(cfg, seed=23)
+    dev = device_tensors(lay)
+    packed = moce.moce_pack_supports(dev["support_idx"], dev["support_logits"], cfg.C_in)
+    pidx, plog, _ = oracle_packed(lay)
+    zref = oracle.pool(lay.x, cfg.layout)
+    zt = torch.from_numpy(zref.astype(np.float32)).cuda()
+    tau, a = moce.moce_gate(zt, packed, dev["W1"], dev["b1"], dev["w2"], dev["b2"], cfg.tau_min,
+                            cfg.tau_max)
+    tref = oracle.gate(zref.astype(np.float32).astype(np.float64), pidx, lay.W1, lay.b1, lay.w2,
+                       float(lay.b2[0]), cfg.tau_min, cfg.tau_max)
+    np.testing.assert_allclose(tau.cpu().numpy(), tref, rtol=2e-5, atol=1e-6)
+    aref = oracle.weights(tau.cpu().numpy().astype(np.float64), plog)
+    np.testing.assert_allclose(a.cpu().numpy(), aref, rtol=2e-5, atol=1e-7)
+
+
 POOL_SHAPES = {
     # (N, H, W, C, dtype, element offset of x): the tilings of the NHWC pool
     "many_spans_c256": (2, 56, 56, 256, "bf16", 0),
