@@ -69,6 +69,9 @@ MUTANTS = {
                                "off += (double)Q[(size_t)(c % R) * d + j] * h[j]"),
     "dynamic_offset_sign": ("Ldyn[((size_t)n * R + e) * C + c] = (double)L[(size_t)e * C + c] + off;",
                             "Ldyn[((size_t)n * R + e) * C + c] = (double)L[(size_t)e * C + c] - off;"),
+    "topk_reads_first_row": ("float v = L[(size_t)e * C + c];", "float v = L[c];"),
+    "topk_off_by_one": ("idx_out[(size_t)e * k + i] = row[i].idx;",
+                        "idx_out[(size_t)e * k + i] = row[i + 1].idx;"),
     "coverage_grad_softmax_jacobian_dot_dropped": ("p[(size_t)e * C + c] * (g[c] - dot) / (double)R;",
                                                    "p[(size_t)e * C + c] * g[c] / (double)R;"),
 }
@@ -78,6 +81,7 @@ PIN_CHECKS = [
     lambda: pins.test_pack_equals_bruteforce_sort(0),
     pins.test_pack_permutation_invariant,
     pins.test_pack_ties_and_signed_zero,
+    pins.test_topk_equals_stable_argsort,
     lambda: pins.test_pack_rejects("dup"),
     lambda: pins.test_cyclic_supports_residual_closed_form(64, 15, 4),
     lambda: pins.test_pool_closed_forms("nhwc"),
