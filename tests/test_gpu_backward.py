@@ -96,6 +96,36 @@ def test_backward_matches_oracle(name):
     _close(g.db2.cpu().numpy(), np.array([ref["db2"]]), "db2")
 
 
+@pytest.mark.parametrize("name", ["rn50_stage1_reduce", "rn50_stage4_reduce"])
+def test_backward_full_size_sampled(name):
+    """The whole workload in the bench's launch configuration. dx of an example depends on that
+    example alone, so sampled examples are compared with the oracle run on the example by itself;
+    the parameter gradients are sums over examples, so the whole batch must give the sum of its
+    two halves' gradients."""
+    from paper_2608_23794_gb300 import moce
+    cfg = CFG[name]
+    lay = synth.make_layer(cfg, seed=5)
+    dyv, dyb = synth.make_dy(cfg, seed=5)
+    dev = device_tensors(lay)
+    dy = torch.from_numpy(dyb.view(np.int16)).view(torch.bfloat16).cuda()
+    packed = moce.moce_pack_supports(dev["support_idx"], dev["support_logits"], cfg.C_in)
+    params = (dev["W1"], dev["b1"], dev["w2"], dev["b2"], cfg.tau_min, cfg.tau_max)
+    g = moce.moce_backward(dev["x"], dy, cfg.layout, packed, *params)
+    h = cfg.N // 2
+    halves = [moce.moce_backward(dev["x"][a:b].contiguous(), dy[a:b].contiguous(), cfg.layout,
+                                 packed, *params) for a, b in ((0, h), (h, cfg.N))]
+    torch.cuda.synchronize()
+    pidx, plog, resid = oracle_packed(lay)
+    for n in (0, h + 1, cfg.N - 1):
+        ref = oracle.backward(lay.x[n:n + 1], dyv[n:n + 1], cfg.layout, pidx, plog, resid, lay.W1,
+                              lay.b1, lay.w2, float(lay.b2[0]), cfg.tau_min, cfg.tau_max)
+        _close(g.dx[n:n + 1].cpu().numpy(), ref["dx"], f"dx of example {n}")
+    for f in ("dlogits", "dW1", "db1", "dw2", "db2"):
+        whole = getattr(g, f).double().cpu().numpy()
+        parts = sum(getattr(q, f).double().cpu().numpy() for q in halves)
+        _close(whole, parts, f"{f}: whole batch against the sum of its halves")
+
+
 def test_backward_is_deterministic():
     from paper_2608_23794_gb300 import moce
     g1, _, (lay, dev, dy, packed) = _run(CASES["rn50_stage3_reduce"])
