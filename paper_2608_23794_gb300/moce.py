@@ -166,8 +166,24 @@ def moce_pack_supports(support_idx: torch.Tensor, support_logits: torch.Tensor, 
     return PackedSupports(out_idx, out_lg, resid, int(n_resid.value), C_in)
 
 
+def moce_status_string(status: int) -> str:
+    return library().moce_status_string(int(status)).decode()
+
+
+def moce_pack_workspace_bytes(C_in: int, C_out: int, k: int) -> int:
+    return int(library().moce_pack_workspace_bytes(C_in, C_out, k))
+
+
 def moce_workspace_bytes(N: int, H: int, W: int, C_in: int, C_out: int, k: int) -> int:
     return int(library().moce_workspace_bytes(N, H, W, C_in, C_out, k))
+
+
+def moce_workspace_offsets(N: int, H: int, W: int, C_in: int, C_out: int, k: int):
+    """Byte offsets of z and tau inside the forward workspace of this shape."""
+    z_off, tau_off = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    _check(library().moce_workspace_offsets(N, H, W, C_in, C_out, k, ctypes.byref(z_off),
+                                            ctypes.byref(tau_off)), "moce_workspace_offsets")
+    return z_off.value, tau_off.value
 
 
 class Workspace:
@@ -179,10 +195,7 @@ class Workspace:
         if nbytes == 0:
             raise MoceError(MOCE_ERR_INVALID_VALUE, "moce_workspace_bytes")
         self.buffer = torch.zeros((nbytes,), dtype=torch.uint8, device=device)
-        z_off, tau_off = ctypes.c_size_t(0), ctypes.c_size_t(0)
-        _check(library().moce_workspace_offsets(N, H, W, C_in, C_out, k, ctypes.byref(z_off),
-                                                ctypes.byref(tau_off)), "moce_workspace_offsets")
-        self.z_offset, self.tau_offset = z_off.value, tau_off.value
+        self.z_offset, self.tau_offset = moce_workspace_offsets(N, H, W, C_in, C_out, k)
 
     @property
     def nbytes(self) -> int:
@@ -197,8 +210,13 @@ class Workspace:
         return self.buffer[self.tau_offset:self.tau_offset + 4 * N * R].view(torch.float32).view(N, R)
 
     def init(self, stream=None):
-        _check(library().moce_workspace_init(_ptr(self.buffer), self.nbytes, _stream(stream)),
-               "moce_workspace_init")
+        moce_workspace_init(self, stream)
+
+
+def moce_workspace_init(ws: Workspace, stream=None):
+    """Zero-fill a forward workspace on the stream (needed again after MOCE_ERR_TIMEOUT)."""
+    _check(library().moce_workspace_init(_ptr(ws.buffer), ws.nbytes, _stream(stream)),
+           "moce_workspace_init")
 
 
 def moce_pool(x: torch.Tensor, layout: str, ws: Workspace | None = None, z=None,
@@ -254,6 +272,22 @@ def moce_forward(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w
     return y
 
 
+def moce_forward_path(x: torch.Tensor, layout: str, packed: PackedSupports, W1, b1, w2, b2,
+                      tau_min: float, tau_max: float, path: str, ws: Workspace | None = None,
+                      y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """moce_forward on the kernel path ``path`` (a key of ``PATHS``)."""
+    return moce_forward(x, layout, packed, W1, b1, w2, b2, tau_min, tau_max, ws=ws, y=y,
+                        stream=stream, path=path)
+
+
+def moce_forward_path_launches(x: torch.Tensor, layout: str, C_out: int, k: int, path: str) -> int:
+    return moce_forward_launches(x, layout, C_out, k, path=path)
+
+
+def moce_forward_path_kernel(x: torch.Tensor, layout: str, C_out: int, k: int, path: str) -> str:
+    return moce_forward_kernel(x, layout, C_out, k, path=path)
+
+
 def moce_forward_launches(x: torch.Tensor, layout: str, C_out: int, k: int,
                           path: str = "auto") -> int:
     """Kernel launches one moce_forward call makes for this input (0: path cannot run it)."""
@@ -302,6 +336,10 @@ def moce_forward_noalloc(x: torch.Tensor, layout: str, packed: PackedSupports, W
                                           float(tau_max), _ptr(y), _stream(stream)),
            "moce_forward_noalloc")
     return y
+
+
+def moce_train_workspace_bytes(C_in: int, C_out: int) -> int:
+    return int(library().moce_train_workspace_bytes(C_in, C_out))
 
 
 def _train_ws(C_in: int, C_out: int, device) -> torch.Tensor:

@@ -36,6 +36,29 @@ def test_every_declared_symbol_is_exported(lib):
         assert hasattr(lib, name), name
 
 
+def test_binding_carries_every_entry_point_by_name(lib):
+    """The Python binding has a function of the same name for every declared entry point; the
+    ones that need no device answer like the library."""
+    from paper_2608_23794_gb300 import moce
+    for name in declared_functions():
+        assert callable(getattr(moce, name, None)), name
+    assert moce.moce_status_string(2) == "MOCE_ERR_BAD_SUPPORT"
+    lib.moce_pack_workspace_bytes.argtypes = [ctypes.c_int] * 3
+    lib.moce_pack_workspace_bytes.restype = ctypes.c_size_t
+    assert moce.moce_pack_workspace_bytes(64, 16, 4) == lib.moce_pack_workspace_bytes(64, 16, 4) > 0
+    assert moce.moce_pack_workspace_bytes(0, 16, 4) == 0
+    assert moce.moce_train_workspace_bytes(256, 64) > 0
+    total = moce.moce_workspace_bytes(2, 8, 8, 64, 16, 4)
+    z_off, tau_off = moce.moce_workspace_offsets(2, 8, 8, 64, 16, 4)
+    assert z_off % 4 == 0 and tau_off % 4 == 0
+    assert z_off + 4 * 2 * 64 <= total and tau_off + 4 * 2 * 16 <= total
+    assert z_off + 4 * 2 * 64 <= tau_off or tau_off + 4 * 2 * 16 <= z_off
+    ws = moce.Workspace(2, 8, 8, 64, 16, 4, device="cpu")  # host buffer: offsets only
+    assert (ws.z_offset, ws.tau_offset, ws.nbytes) == (z_off, tau_off, total)
+    with pytest.raises(ValueError):  # the library is never handed a host buffer
+        moce.moce_workspace_init(ws)
+
+
 def test_status_strings(lib):
     lib.moce_status_string.restype = ctypes.c_char_p
     lib.moce_status_string.argtypes = [ctypes.c_int]
